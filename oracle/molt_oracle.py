@@ -1,0 +1,248 @@
+"""fp64 CPU oracle for the per-token policy-update path of MOLT (arxiv 2607.21653).
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, the smoke check of the package entry
+file and the CPU-baseline leg of the benchmark may import this module.  It
+shares no code with the CUDA library and imports nothing from it.
+
+Every function is a plain restatement of a definition, in fp64, applied to the
+exact bits the GPU reads (bf16 hidden states and weights widened exactly).
+Library primitives used as steps: numpy matmul (the LM-head product), exp/log.
+There is no blocking, fusion or reordering beyond splitting rows into blocks
+to bound memory, which does not change any per-element result.
+
+What the paper fixes and what is a stated reading (the paper describes the
+method at framework level only):
+
+* Group advantage (Sec. 4.5: GRPO among the estimators; Sec. 4.2: a rollout's
+  reward is counted once and mapped back to its segments).  Reading: per
+  contiguous prompt group, A_j = (r_j - mean) / (std + eps) with the unbiased
+  (n-1) standard deviation, eps = 1e-6 added outside the square root, a group of
+  one response gets A = 0, and a zero-variance group gets exactly 0.  The fp64
+  sums run in index order; the result is rounded once to fp32.
+* Recomputed log-probabilities (Sec. 4.5, "the actor's recomputed
+  probabilities"): z = h W^T, lse = log sum exp z, logp = z[x] - lse.
+* Entropy (not in the paper; part of the hot path's forward outputs): Shannon
+  entropy of softmax(z) in nats, H = lse - sum_v p_v z_v.  No gradient.
+* Importance ratio against recorded behaviour log-probs (Sec. 4.3, Sec. 4.5):
+  rho = exp(logp - b).
+* Clipped surrogate (Sec. 4.5 "masking and clipping"; PPO is the cited
+  objective).  Reading: l = -min(rho*A, clip(rho, 1-eps_lo, 1+eps_hi)*A), with
+  asymmetric clip bounds and no KL, entropy bonus or dual clip.  The clipped
+  branch is selected when (A>0 and rho>1+eps_hi) or (A<0 and rho<1-eps_lo),
+  which is the same minimum written as a rule; ties count as unclipped.
+* Token-mean normalisation, Eq. 2: L = sum_i m_i l_i / D with one denominator D
+  for the whole optimizer window; D defaults to sum_i m_i of the call.
+* Backward: dL/dz_tv = (m_t / D) c_t (p_tv - [v == x_t]) with c_t = rho_t A_t on
+  the unclipped branch and 0 on the clipped one; dH = G W, dW = G^T h.
+
+Pins (tests/test_oracle.py): closed-form advantages, zero/one-response groups,
+library log_softmax / entropy, sum exp(logp) = 1, the rho = 1 case against the
+autograd gradient of advantage-weighted cross-entropy, clipped rows having zero
+gradient, special clip values, finite differences of the loss, microbatch-split
+invariance of Eq. 2 and segment-split invariance of the advantages.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+__all__ = [
+    "widen_bf16", "group_advantages", "broadcast_advantages", "logits_rows",
+    "row_softmax_stats", "token_logprobs", "policy_loss", "policy_loss_rows",
+    "clip_decision", "surrogate",
+]
+
+DEFAULT_ADV_EPS = 1e-6
+
+
+def widen_bf16(bits: np.ndarray) -> np.ndarray:
+    """bf16 bit pattern -> fp64 value (exact)."""
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return u.view(np.float32).astype(np.float64)
+
+
+# --------------------------------------------------------------------------- #
+# Advantages (Sec. 4.5 GRPO; Sec. 4.2 segments share the rollout reward)
+# --------------------------------------------------------------------------- #
+def group_advantages(rewards: np.ndarray, group_ids: np.ndarray,
+                     eps: float = DEFAULT_ADV_EPS) -> np.ndarray:
+    """GRPO group-normalised advantage per response, groups = maximal runs of
+    equal consecutive ids.  Plain fp64 loops in index order; each operation is
+    one correctly rounded IEEE double operation, result rounded to fp32."""
+    r = np.asarray(rewards, dtype=np.float32)
+    g = np.asarray(group_ids)
+    n = r.shape[0]
+    out = np.zeros(n, dtype=np.float32)
+    start = 0
+    while start < n:
+        end = start + 1
+        while end < n and g[end] == g[start]:
+            end += 1
+        cnt = end - start
+        if cnt > 1:
+            s = 0.0
+            for j in range(start, end):
+                s = s + float(r[j])
+            mean = s / float(cnt)
+            ss = 0.0
+            for j in range(start, end):
+                d = float(r[j]) - mean
+                ss = ss + d * d
+            std = math.sqrt(ss / float(cnt - 1))
+            den = std + eps
+            for j in range(start, end):
+                out[j] = np.float32((float(r[j]) - mean) / den)
+        start = end
+    return out
+
+
+def broadcast_advantages(adv_resp: np.ndarray, resp_of_token: np.ndarray) -> np.ndarray:
+    """Per-token advantage = advantage of the rollout the token belongs to."""
+    return np.asarray(adv_resp, dtype=np.float32)[np.asarray(resp_of_token)]
+
+
+# --------------------------------------------------------------------------- #
+# Log-softmax, gather, entropy (Sec. 4.5 recomputed probabilities)
+# --------------------------------------------------------------------------- #
+def logits_rows(h_rows: np.ndarray, W: np.ndarray) -> np.ndarray:
+    """z = h W^T for a block of rows (fp64)."""
+    return h_rows @ W.T
+
+
+def row_softmax_stats(z: np.ndarray, x: np.ndarray):
+    """For each row of z: lse, logp of target x, entropy, probabilities p."""
+    M = z.max(axis=1, keepdims=True)
+    e = np.exp(z - M)
+    ssum = e.sum(axis=1, keepdims=True)
+    lse = (M + np.log(ssum))[:, 0]
+    p = np.exp(z - lse[:, None])
+    logp = z[np.arange(z.shape[0]), x] - lse
+    ent = lse - (p * z).sum(axis=1)
+    return lse, logp, ent, p
+
+
+def token_logprobs(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, mask: np.ndarray | None,
+                   rows: np.ndarray | None = None, block: int = 64):
+    """logp and entropy per token (fp64).  `hidden`/`W` are fp64 (use widen_bf16
+    on bf16 bits).  Rows with mask 0 are not computed and return 0.  If `rows`
+    is given, only those row indices are computed (returned in that order)."""
+    T = hidden.shape[0]
+    idx = np.arange(T) if rows is None else np.asarray(rows)
+    logp = np.zeros(idx.shape[0])
+    ent = np.zeros(idx.shape[0])
+    act = np.ones(idx.shape[0], dtype=bool) if mask is None else (np.asarray(mask)[idx] != 0)
+    sel = np.nonzero(act)[0]
+    for b0 in range(0, sel.shape[0], block):
+        k = sel[b0:b0 + block]
+        t = idx[k]
+        z = logits_rows(hidden[t], W)
+        _, lp, en, _ = row_softmax_stats(z, np.asarray(tokens)[t])
+        logp[k] = lp
+        ent[k] = en
+    return logp, ent
+
+
+# --------------------------------------------------------------------------- #
+# Ratio, clipped surrogate, Eq. 2 normalisation and the backward pass
+# --------------------------------------------------------------------------- #
+def clip_decision(rho: np.ndarray, adv: np.ndarray, eps_lo: float, eps_hi: float) -> np.ndarray:
+    """True where the clipped term of min(rho*A, clip(rho)*A) is the smaller one."""
+    lo = 1.0 - float(eps_lo)
+    hi = 1.0 + float(eps_hi)
+    return ((adv > 0) & (rho > hi)) | ((adv < 0) & (rho < lo))
+
+
+def surrogate(rho: np.ndarray, adv: np.ndarray, eps_lo: float, eps_hi: float):
+    """Per-token loss l = -min(rho A, clip(rho) A) and its derivative coefficient
+    c = -dl/dlogp (rho A on the unclipped branch, 0 on the clipped one)."""
+    lo = 1.0 - float(eps_lo)
+    hi = 1.0 + float(eps_hi)
+    clipped = clip_decision(rho, adv, eps_lo, eps_hi)
+    rho_c = np.minimum(np.maximum(rho, lo), hi)
+    loss = np.where(clipped, -rho_c * adv, -rho * adv)
+    coef = np.where(clipped, 0.0, rho * adv)
+    return loss, coef, clipped
+
+
+def policy_loss_rows(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray,
+                     behavior_logp: np.ndarray, adv: np.ndarray, mask: np.ndarray,
+                     eps_lo: float, eps_hi: float, denom: float, rows: np.ndarray,
+                     want_dW: bool = False, block: int = 64):
+    """Per-row forward quantities and dH rows for the given row indices.
+
+    Returns dict with logp, entropy, lse, ratio, token_loss (m*l), coef
+    (m*c/D), clipped, dH (len(rows) x H) and, if want_dW, the contribution of
+    these rows to dW (V x H).  Each row is independent of the others, so this
+    is exactly the corresponding slice of the full computation."""
+    rows = np.asarray(rows)
+    n = rows.shape[0]
+    H = hidden.shape[1]
+    out = {k: np.zeros(n) for k in ("logp", "entropy", "lse", "ratio", "token_loss", "coef")}
+    out["clipped"] = np.zeros(n, dtype=bool)
+    out["dH"] = np.zeros((n, H))
+    dW = np.zeros_like(W) if want_dW else None
+    m_all = np.asarray(mask).astype(np.float64)
+    for b0 in range(0, n, block):
+        sl = slice(b0, min(n, b0 + block))
+        t = rows[sl]
+        m = m_all[t]
+        act = m != 0
+        if not act.any():
+            continue
+        t_a = t[act]
+        pos = np.arange(sl.start, sl.stop)[act]
+        h_a = hidden[t_a]
+        x = np.asarray(tokens)[t_a]
+        z = logits_rows(h_a, W)
+        lse, logp, ent, p = row_softmax_stats(z, x)
+        rho = np.exp(logp - np.asarray(behavior_logp, dtype=np.float64)[t_a])
+        a = np.asarray(adv, dtype=np.float64)[t_a]
+        loss, c, clipped = surrogate(rho, a, eps_lo, eps_hi)
+        coef = c / denom                       # m = 1 on these rows
+        g = coef[:, None] * p
+        g[np.arange(g.shape[0]), x] -= coef
+        out["logp"][pos] = logp
+        out["entropy"][pos] = ent
+        out["lse"][pos] = lse
+        out["ratio"][pos] = rho
+        out["token_loss"][pos] = loss
+        out["coef"][pos] = coef
+        out["clipped"][pos] = clipped
+        out["dH"][pos] = g @ W
+        if want_dW:
+            dW += g.T @ h_a
+    out["dW"] = dW
+    return out
+
+
+def policy_loss(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, behavior_logp: np.ndarray,
+                adv: np.ndarray, mask: np.ndarray, eps_lo: float, eps_hi: float,
+                denom: float | None = None, block: int = 64):
+    """Full fp64 forward + backward of the token-mean clipped surrogate (Eq. 2).
+
+    hidden [T,H] and W [V,H] are fp64; adv is the per-token advantage.  Returns
+    loss, per-token quantities (masked rows 0), dH [T,H], dW [V,H] and the
+    window statistics."""
+    T = hidden.shape[0]
+    m = np.asarray(mask).astype(np.float64)
+    D = float(m.sum()) if (denom is None or denom <= 0) else float(denom)
+    if D == 0.0:
+        raise ZeroDivisionError("Eq. 2 needs a nonzero denominator")
+    r = policy_loss_rows(hidden, W, tokens, behavior_logp, adv, mask, eps_lo, eps_hi, D,
+                         np.arange(T), want_dW=True, block=block)
+    loss = float(r["token_loss"].sum() / D)
+    act = m != 0
+    a = np.asarray(adv, dtype=np.float64)
+    n_act = int(act.sum())
+    stats = {
+        "n_active": n_act,
+        "loss": loss,
+        "clip_frac_low": float(((r["clipped"]) & (a < 0) & act).sum() / max(1, n_act)),
+        "clip_frac_high": float(((r["clipped"]) & (a > 0) & act).sum() / max(1, n_act)),
+        "mean_ratio": float(r["ratio"][act].mean()) if n_act else 0.0,
+        "mean_entropy": float(r["entropy"][act].mean()) if n_act else 0.0,
+        "max_abs_log_ratio": float(np.abs(np.log(r["ratio"][act])).max()) if n_act else 0.0,
+    }
+    r.update(loss=loss, denom=D, stats=stats)
+    return r

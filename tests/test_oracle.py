@@ -1,0 +1,270 @@
+"""Pins for the fp64 oracle, against things other than the oracle itself:
+hand-derived values, closed forms, library routines (scipy log_softmax /
+entropy, torch autograd of cross-entropy), finite differences and the
+invariances that Eq. 2 and the segment rule of Sec. 4.2 state."""
+import math
+
+import numpy as np
+import pytest
+import scipy.special
+import scipy.stats
+
+from oracle import molt_oracle as O
+from workloads import bf16_bits_to_f32, f32_to_bf16_bits, make_workload
+
+GOLDEN = __import__("os").path.join(__import__("os").path.dirname(__file__), "golden")
+
+
+def _read_golden(name):
+    rows = []
+    with open(f"{GOLDEN}/{name}") as f:
+        for line in f:
+            line = line.split("#", 1)[0].strip()
+            if line:
+                rows.append(line)
+    return rows
+
+
+# ----------------------------------------------------------------- advantages
+def test_advantages_hand_values():
+    """Hand-derived GRPO values (tests/golden/grpo_hand.txt)."""
+    for row in _read_golden("grpo_hand.txt"):
+        rs, want = row.split("|")
+        r = np.array([float(v) for v in rs.split()], dtype=np.float32)
+        want = np.array([float(v) for v in want.split()], dtype=np.float64)
+        got = O.group_advantages(r, np.zeros(len(r), dtype=np.int32))
+        np.testing.assert_array_equal(got, want.astype(np.float32), err_msg=row)
+
+
+def test_advantages_degenerate_groups():
+    r = np.array([0.3, 0.3, 0.3, 0.3, 7.0, 1.0, 1.0], dtype=np.float32)
+    g = np.array([0, 0, 0, 0, 1, 2, 2], dtype=np.int32)
+    a = O.group_advantages(r, g)
+    assert (a == 0).all()          # zero-variance groups and a one-response group give exactly 0
+
+
+def test_advantages_match_library_and_moments():
+    rng = np.random.default_rng(11)
+    for G in (2, 3, 4, 8, 16, 33, 64):
+        r = rng.random(G).astype(np.float32)
+        a = O.group_advantages(r, np.zeros(G, dtype=np.int32))
+        r64 = r.astype(np.float64)
+        ref = (r64 - r64.mean()) / (r64.std(ddof=1) + 1e-6)
+        np.testing.assert_allclose(a, ref.astype(np.float32), rtol=2e-7, atol=1e-7)
+        assert abs(float(a.astype(np.float64).sum())) < 1e-5 * G
+        sd = r64.std(ddof=1)
+        assert abs(a.astype(np.float64).std(ddof=1) - sd / (sd + 1e-6)) < 1e-5
+
+
+def test_advantages_groups_are_independent_and_permute():
+    rng = np.random.default_rng(3)
+    r = rng.random(40).astype(np.float32)
+    g = np.repeat(np.arange(5), 8).astype(np.int32)
+    a = O.group_advantages(r, g)
+    for k in range(5):
+        np.testing.assert_array_equal(a[8 * k:8 * k + 8],
+                                      O.group_advantages(r[8 * k:8 * k + 8], np.zeros(8, np.int32)))
+    perm = np.array([3, 0, 4, 1, 2])
+    rp = np.concatenate([r[8 * k:8 * k + 8] for k in perm])
+    ap = O.group_advantages(rp, g)
+    np.testing.assert_array_equal(ap, np.concatenate([a[8 * k:8 * k + 8] for k in perm]))
+
+
+def test_segment_split_invariance():
+    """Sec. 4.2: segments of one rollout share its reward, counted once."""
+    w = make_workload("long_traj", with_tensors=False, T=8 * 512)
+    a_resp = O.group_advantages(w.rewards, w.group_ids)
+    a_tok = O.broadcast_advantages(a_resp, w.resp_of_token)
+    seg = w.extra["segment_of_token"]
+    for s in np.unique(seg):
+        toks = np.nonzero(seg == s)[0]
+        assert np.unique(a_tok[toks]).size == 1
+        assert a_tok[toks[0]] == a_resp[w.resp_of_token[toks[0]]]
+    # the same rewards without any split give the same advantages
+    np.testing.assert_array_equal(a_resp, O.group_advantages(w.rewards, np.zeros(8, np.int32)))
+
+
+# ----------------------------------------------------------- log-softmax etc.
+def test_logprobs_sum_to_one_and_match_library():
+    rng = np.random.default_rng(5)
+    T, H, V = 6, 9, 13
+    h = rng.standard_normal((T, H))
+    W = rng.standard_normal((V, H)) * 0.7
+    z = h @ W.T
+    tot = np.zeros(T)
+    for v in range(V):
+        lp, ent = O.token_logprobs(h, W, np.full(T, v), None)
+        tot += np.exp(lp)
+        np.testing.assert_allclose(lp, scipy.special.log_softmax(z, axis=1)[:, v], rtol=0, atol=1e-12)
+        p = scipy.special.softmax(z, axis=1)
+        np.testing.assert_allclose(ent, scipy.stats.entropy(p, axis=1), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(tot, 1.0, rtol=0, atol=1e-12)
+
+
+def test_uniform_logits_closed_form():
+    T, H, V = 4, 8, 1000
+    h = np.ones((T, H))
+    W = np.zeros((V, H))
+    lp, ent = O.token_logprobs(h, W, np.arange(T), None)
+    np.testing.assert_allclose(lp, -math.log(V), atol=1e-13)
+    np.testing.assert_allclose(ent, math.log(V), atol=1e-13)
+
+
+def test_masked_rows_zero():
+    rng = np.random.default_rng(2)
+    h = rng.standard_normal((5, 4))
+    W = rng.standard_normal((7, 4))
+    mask = np.array([1, 0, 1, 0, 0], np.uint8)
+    lp, ent = O.token_logprobs(h, W, np.arange(5) % 7, mask)
+    assert (lp[mask == 0] == 0).all() and (ent[mask == 0] == 0).all()
+    assert (lp[mask == 1] < 0).all()
+
+
+def test_bf16_widening_exact():
+    x = np.array([1.0, -2.5, 3.140625, 1e-3, 65504.0], dtype=np.float32)
+    bits = f32_to_bf16_bits(x)
+    np.testing.assert_array_equal(O.widen_bf16(bits), bf16_bits_to_f32(bits).astype(np.float64))
+    assert O.widen_bf16(np.array([0x3F80], np.uint16))[0] == 1.0
+    assert O.widen_bf16(np.array([0xC020], np.uint16))[0] == -2.5
+
+
+# ---------------------------------------------------------- clipped surrogate
+def _small_problem(seed, T=8, H=16, V=32, mask=None):
+    rng = np.random.default_rng(seed)
+    h = rng.standard_normal((T, H))
+    W = rng.standard_normal((V, H)) * 0.3
+    x = rng.integers(0, V, T)
+    m = np.ones(T, np.uint8) if mask is None else np.asarray(mask, np.uint8)
+    return h, W, x, m
+
+
+def test_clip_special_values():
+    """Hand values of l = -min(rho A, clip(rho) A) for chosen rho."""
+    h, W, x, m = _small_problem(0, T=6)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    rho = np.array([1.0, 1.5, 0.5, 0.5, 1.5, 1.1])
+    adv = np.array([0.7, 2.0, -1.0, 3.0, -0.5, -2.0])
+    b = lp - np.log(rho)
+    r = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.28)
+    want_l = np.array([-0.7, -1.28 * 2.0, -0.8 * -1.0, -0.5 * 3.0, -1.5 * -0.5, -1.1 * -2.0])
+    want_clip = np.array([False, True, True, False, False, False])
+    np.testing.assert_allclose(r["token_loss"], want_l, rtol=1e-12)
+    np.testing.assert_array_equal(r["clipped"], want_clip)
+    assert (r["dH"][want_clip] == 0).all()
+    assert np.abs(r["dH"][~want_clip]).max() > 0
+    np.testing.assert_allclose(r["loss"], want_l.sum() / 6, rtol=1e-12)
+
+
+def test_rho_one_equals_weighted_nll_gradient():
+    """At rho = 1 the gradient is that of sum m A CE(z, x) / D (torch autograd)."""
+    torch = pytest.importorskip("torch")
+    h, W, x, m = _small_problem(1, T=10, H=12, V=20, mask=[1, 1, 0, 1, 1, 1, 0, 1, 1, 1])
+    adv = np.random.default_rng(9).standard_normal(10)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    r = O.policy_loss(h, W, x, lp, adv, m, 0.2, 0.2)
+    th = torch.tensor(h, requires_grad=True)
+    tW = torch.tensor(W, requires_grad=True)
+    ce = torch.nn.functional.cross_entropy(th @ tW.T, torch.tensor(x), reduction="none")
+    L = (torch.tensor(m, dtype=torch.float64) * torch.tensor(adv) * ce).sum() / float(m.sum())
+    L.backward()
+    np.testing.assert_allclose(r["dH"], th.grad.numpy(), rtol=1e-10, atol=1e-13)
+    np.testing.assert_allclose(r["dW"], tW.grad.numpy(), rtol=1e-10, atol=1e-13)
+    np.testing.assert_allclose(r["loss"], -(m * adv).sum() / m.sum(), rtol=1e-12)
+
+
+def test_full_gradient_matches_autograd():
+    """Independent derivation of the backward: torch autograd of the surrogate."""
+    torch = pytest.importorskip("torch")
+    h, W, x, m = _small_problem(4, T=12, H=10, V=24, mask=[1] * 9 + [0] * 3)
+    rng = np.random.default_rng(8)
+    adv = rng.standard_normal(12)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    b = lp + rng.choice([-0.6, -0.1, 0.05, 0.4], size=12)
+    D = 17.0
+    r = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.28, denom=D)
+    th = torch.tensor(h, requires_grad=True)
+    tW = torch.tensor(W, requires_grad=True)
+    logp = torch.log_softmax(th @ tW.T, dim=1)[torch.arange(12), torch.tensor(x)]
+    rho = torch.exp(logp - torch.tensor(b))
+    A = torch.tensor(adv)
+    l = -torch.minimum(rho * A, torch.clamp(rho, 0.8, 1.28) * A)
+    L = (torch.tensor(m, dtype=torch.float64) * l).sum() / D
+    L.backward()
+    np.testing.assert_allclose(r["loss"], L.item(), rtol=1e-12)
+    np.testing.assert_allclose(r["dH"], th.grad.numpy(), rtol=1e-9, atol=1e-13)
+    np.testing.assert_allclose(r["dW"], tW.grad.numpy(), rtol=1e-9, atol=1e-13)
+
+
+def test_finite_differences():
+    h, W, x, m = _small_problem(7, T=8, H=16, V=32, mask=[1, 1, 1, 0, 1, 1, 1, 1])
+    rng = np.random.default_rng(1)
+    adv = rng.standard_normal(8)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    b = lp - np.log(np.array([1.0, 1.5, 0.5, 1.0, 0.9, 1.1, 0.6, 1.4]))
+    r = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.2)
+    step = 1e-6
+
+    def f(hh, WW):
+        return O.policy_loss(hh, WW, x, b, adv, m, 0.2, 0.2)["loss"]
+
+    gh = np.zeros_like(h)
+    for i in range(h.shape[0]):
+        for j in range(h.shape[1]):
+            hp, hm = h.copy(), h.copy()
+            hp[i, j] += step
+            hm[i, j] -= step
+            gh[i, j] = (f(hp, W) - f(hm, W)) / (2 * step)
+    gW = np.zeros_like(W)
+    for i in range(W.shape[0]):
+        for j in range(W.shape[1]):
+            Wp, Wm = W.copy(), W.copy()
+            Wp[i, j] += step
+            Wm[i, j] -= step
+            gW[i, j] = (f(h, Wp) - f(h, Wm)) / (2 * step)
+    np.testing.assert_allclose(r["dH"], gh, rtol=1e-5, atol=1e-9)
+    np.testing.assert_allclose(r["dW"], gW, rtol=1e-5, atol=1e-9)
+
+
+def test_microbatch_split_invariance():
+    """Eq. 2: with one window denominator, microbatch losses/gradients add up."""
+    h, W, x, m = _small_problem(12, T=20, H=8, V=16, mask=[1, 0, 1, 1, 1] * 4)
+    rng = np.random.default_rng(12)
+    adv = rng.standard_normal(20)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    b = lp + rng.normal(0, 0.2, 20)
+    full = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.2)
+    D = full["denom"]
+    parts = [slice(0, 7), slice(7, 8), slice(8, 20)]
+    tot, dW = 0.0, np.zeros_like(W)
+    for s in parts:
+        p = O.policy_loss(h[s], W, x[s], b[s], adv[s], m[s], 0.2, 0.2, denom=D)
+        tot += p["loss"]
+        dW += p["dW"]
+        np.testing.assert_allclose(p["dH"], full["dH"][s], rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(tot, full["loss"], rtol=1e-12)
+    np.testing.assert_allclose(dW, full["dW"], rtol=1e-11, atol=1e-15)
+
+
+def test_gradient_row_and_column_sums_vanish():
+    """sum_v g_tv = 0 per token, hence sum_v dW[v,:] = 0 (closed form)."""
+    h, W, x, m = _small_problem(13, T=16, H=8, V=40)
+    rng = np.random.default_rng(13)
+    adv = rng.standard_normal(16)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    r = O.policy_loss(h, W, x, lp + rng.normal(0, .1, 16), adv, m, 0.2, 0.2)
+    np.testing.assert_allclose(r["dW"].sum(axis=0), 0.0, atol=1e-13)
+    # trace identity: sum_t <dH_t, h_t> = sum_v <dW_v, W_v>
+    np.testing.assert_allclose((r["dH"] * h).sum(), (r["dW"] * W).sum(), rtol=1e-10)
+
+
+def test_rows_subset_equals_full():
+    h, W, x, m = _small_problem(14, T=30, H=8, V=12, mask=[1, 1, 0] * 10)
+    rng = np.random.default_rng(14)
+    adv = rng.standard_normal(30)
+    b = rng.normal(-2.5, 0.5, 30)
+    full = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.2)
+    rows = np.array([29, 3, 4, 17, 0])
+    sub = O.policy_loss_rows(h, W, x, b, adv, m, 0.2, 0.2, full["denom"], rows)
+    for k in ("logp", "entropy", "ratio", "token_loss", "coef"):
+        np.testing.assert_array_equal(sub[k], full[k][rows])
+    np.testing.assert_allclose(sub["dH"], full["dH"][rows], rtol=1e-13, atol=1e-16)
