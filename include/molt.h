@@ -1,0 +1,161 @@
+/*
+ * molt.h — C ABI of the GB300 (sm_103a) policy-update hot path of MOLT
+ * (arxiv 2607.21653): GRPO group advantages, the LM-head log-probability /
+ * entropy forward, and the fused clipped-surrogate forward + backward with the
+ * token-mean normalisation of Eq. 2.
+ *
+ * Conventions shared by every call
+ *   - All array pointers are DEVICE pointers owned by the caller; the library
+ *     never frees them.  bf16 tensors are passed as their 16-bit patterns
+ *     (uint16_t), row-major, 16-byte aligned.
+ *   - Calls are asynchronous on `stream`.  Arguments are validated on the host
+ *     before anything is launched; a non-OK return means nothing was launched
+ *     and no output was written.  The thread-local molt_last_error() explains
+ *     the last non-OK return.
+ *   - Conditions that only the device can see (a token id out of range on an
+ *     active row, a zero token count when the denominator is taken from the
+ *     mask, unsorted group ids, a pipeline wait that timed out) set bits of a
+ *     per-device status word that molt_device_status() reads and clears.
+ *   - Workspace: calls that need scratch memory take (workspace, bytes).  The
+ *     size comes from the matching *_workspace_bytes() query.  Passing NULL
+ *     makes the call allocate and free it stream-ordered (cudaMallocAsync).
+ *   - The library keeps no state between calls except cached device properties
+ *     and the per-device status word; it is safe to call from several threads
+ *     on different streams with different workspaces.
+ */
+#ifndef MOLT_H_
+#define MOLT_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  MOLT_OK = 0,
+  MOLT_ERR_INVALID_ARG = 1,       /* null / misaligned pointer, negative size, bad clip range */
+  MOLT_ERR_UNSUPPORTED_SHAPE = 2, /* H not a positive multiple of 64, or a size beyond int32 */
+  MOLT_ERR_UNSORTED_GROUPS = 3,   /* (device status) group ids decrease somewhere */
+  MOLT_ERR_ZERO_DENOM = 4,        /* (device status) Eq. 2 denominator is zero */
+  MOLT_ERR_CUDA = 5,              /* a CUDA runtime/driver call failed */
+  MOLT_ERR_DEVICE_TIMEOUT = 6,    /* (device status) a pipeline wait gave up */
+  MOLT_ERR_NO_MEMORY = 7,         /* workspace allocation failed */
+  MOLT_ERR_TOKEN_RANGE = 8,       /* (device status) tokens[t] outside [0, V) on an active row */
+  MOLT_ERR_WORKSPACE = 9          /* caller workspace smaller than *_workspace_bytes() */
+} molt_status;
+
+/* bits of the device status word */
+#define MOLT_DEV_TIMEOUT 1u
+#define MOLT_DEV_TOKEN_RANGE 2u
+#define MOLT_DEV_ZERO_DENOM 4u
+#define MOLT_DEV_UNSORTED_GROUPS 8u
+
+/* Window statistics written (device memory) by molt_policy_loss_fwd_bwd.
+ * Counts and sums run over active (mask = 1) tokens of this call. */
+typedef struct {
+  double denom;             /* D actually used in Eq. 2 */
+  double loss;              /* sum_i m_i l_i / D */
+  double sum_ratio;         /* sum of rho_i */
+  double sum_entropy;       /* sum of per-token entropies (nats) */
+  double max_abs_log_ratio; /* max |logp_i - b_i| */
+  int64_t n_active;         /* sum_i m_i */
+  int64_t n_clip_low;       /* tokens on the clipped branch with A_i < 0 (rho < 1 - eps_lo) */
+  int64_t n_clip_high;      /* tokens on the clipped branch with A_i > 0 (rho > 1 + eps_hi) */
+} molt_stats;
+
+const char* molt_status_string(molt_status s);
+/* Text of the last non-OK status returned on the calling thread. */
+const char* molt_last_error(void);
+int molt_version(void);
+
+/* Synchronises `stream`, returns the current device's status word in *flags
+ * (MOLT_DEV_* bits) and clears it.  Returns the molt_status of the highest
+ * priority set bit (MOLT_OK if none). */
+molt_status molt_device_status(cudaStream_t stream, uint32_t* flags);
+
+/*
+ * GRPO group-normalised advantages (Sec. 4.5 lists GRPO among the advantage
+ * estimators; Sec. 4.2: segments of one rollout share its reward, which group
+ * estimators count once).
+ *   rewards   [n_resp] fp32, one reward per rollout (not per segment)
+ *   group_ids [n_resp] int32, non-decreasing; a prompt group is a maximal
+ *             run of equal consecutive ids.  An id smaller than its
+ *             predecessor sets MOLT_DEV_UNSORTED_GROUPS (each run is still
+ *             normalised on its own).
+ *   eps       added to the unbiased (n-1) standard deviation
+ *   adv_out   [n_resp] fp32: A_j = (r_j - mean_g) / (std_g + eps); groups of one
+ *             response and zero-variance groups give exactly 0.
+ * Arithmetic is fp64 in index order with correctly rounded operations, so the
+ * result is bit-identical to a sequential fp64 evaluation rounded to fp32.
+ */
+molt_status molt_group_advantages(const float* rewards, const int32_t* group_ids, int64_t n_resp, double eps,
+                                  float* adv_out, cudaStream_t stream);
+
+/* Per-token advantages: adv_tok[t] = adv_resp[resp_of_token[t]] (Sec. 4.2: the
+ * rollout-level result is mapped back to its segments' tokens).
+ * resp_of_token [T] int32 in [0, n_resp); out-of-range ids give 0. */
+molt_status molt_broadcast_advantages(const float* adv_resp, const int32_t* resp_of_token, int64_t n_resp,
+                                      int64_t T, float* adv_tok, cudaStream_t stream);
+
+/* Number of active tokens sum_i m_i (the Eq. 2 denominator of one call),
+ * written as an int64 to device memory `count_out`.  mask [T] uint8 (0/1). */
+molt_status molt_mask_count(const uint8_t* mask, int64_t T, int64_t* count_out, cudaStream_t stream);
+
+/*
+ * Recomputed log-probabilities and entropies of the generated tokens
+ * (Sec. 4.5: the actor's recomputed probabilities), without materialising the
+ * [T, V] logits:
+ *   z_tv = sum_k hidden[t,k] W[v,k];  lse_t = log sum_v exp z_tv
+ *   logp_out[t] = z_{t,tokens[t]} - lse_t
+ *   entropy_out[t] = lse_t - sum_v softmax(z_t)_v z_tv        (nats)
+ *   hidden [T,H] bf16, W [V,H] bf16 (nn.Linear layout), tokens [T] int32,
+ *   mask [T] uint8 or NULL (= all active).  Rows with mask 0 are skipped and
+ *   their outputs are 0.  entropy_out may be NULL.
+ * Shapes: T >= 0, V >= 1, H a positive multiple of 64, T, V < 2^31.
+ * bf16 products accumulate in fp32 on the tensor cores; outputs are fp32.
+ */
+size_t molt_token_logprobs_workspace_bytes(int64_t T, int64_t H, int64_t V);
+molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                                    const uint8_t* mask, int64_t T, int64_t H, int64_t V, float* logp_out,
+                                    float* entropy_out, void* workspace, size_t workspace_bytes,
+                                    cudaStream_t stream);
+
+/*
+ * Fused clipped-surrogate policy loss with Eq. 2 normalisation, forward and
+ * backward (Sec. 4.5):
+ *   rho_t = exp(logp_t - behavior_logp[t])                 importance ratio
+ *   l_t   = -min(rho_t A_t, clip(rho_t, 1 - clip_lo, 1 + clip_hi) A_t)
+ *   loss  = sum_t m_t l_t / D,  D = denom if denom > 0, else sum_t m_t
+ *   dL/dz_tv = (m_t / D) c_t (softmax(z_t)_v - [v == tokens[t]]),
+ *              c_t = rho_t A_t on the unclipped branch, 0 on the clipped one
+ *   dhidden = dL/dz W   [T,H] bf16 (rows with mask 0 are exactly 0)
+ *   dW     (+)= dL/dz^T hidden   [V,H] fp32; accumulate_dW = 0 overwrites,
+ *              1 adds to the caller's buffer (microbatches of one window).
+ * Inputs: hidden [T,H] bf16, W [V,H] bf16, tokens [T] int32, behavior_logp [T]
+ * fp32, adv [T] fp32 per-token advantages, mask [T] uint8 or NULL.
+ * Use one window-wide `denom` for every microbatch of an optimizer window
+ * (Eq. 2); with denom <= 0 and no active token the loss and gradients are 0
+ * and MOLT_DEV_ZERO_DENOM is set.
+ * Outputs: loss_out (device fp32 scalar), dhidden_out, dW_out; optional
+ * (may be NULL): logp_out [T], entropy_out [T], token_loss_out [T] (= m_t l_t),
+ * stats_out (device molt_stats).
+ * The [T,V] logits and gradients never reach global memory: each vocab tile is
+ * recomputed on chip in the backward pass and fed to the dhidden / dW tensor-
+ * core products from shared memory.
+ */
+size_t molt_policy_loss_workspace_bytes(int64_t T, int64_t H, int64_t V);
+molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                                     const float* behavior_logp, const float* adv, const uint8_t* mask,
+                                     int64_t T, int64_t H, int64_t V, float clip_lo, float clip_hi,
+                                     double denom, float* loss_out, uint16_t* dhidden_out, float* dW_out,
+                                     int accumulate_dW, float* logp_out, float* entropy_out,
+                                     float* token_loss_out, molt_stats* stats_out, void* workspace,
+                                     size_t workspace_bytes, cudaStream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MOLT_H_ */

@@ -1,0 +1,293 @@
+"""Python binding of libmolt: the GB300 (sm_103a) policy-update hot path of
+MOLT (arxiv 2607.21653).
+
+Every function here only marshals arguments into the C ABI declared in
+include/molt.h: torch CUDA tensors become raw device pointers, the current CUDA
+stream is passed along, and every step runs in the library's CUDA kernels.
+There is no CPU fallback: if the library is not built, or a tensor is not on a
+CUDA device, the call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import subprocess
+import sys
+from concurrent.futures import ThreadPoolExecutor
+
+__all__ = [
+    "build", "load", "lib_path", "MoltError", "STATUS", "DEV_FLAGS", "group_advantages",
+    "broadcast_advantages", "mask_count", "token_logprobs", "policy_loss_fwd_bwd", "device_status",
+    "token_logprobs_workspace_bytes", "policy_loss_workspace_bytes", "header_functions",
+]
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+_ROOT = os.path.dirname(_PKG)
+_CSRC = os.path.join(_PKG, "csrc")
+_INCLUDE = os.path.join(_ROOT, "include")
+_BUILD = os.path.join(_ROOT, "_build")
+_LIB = os.path.join(_PKG, "libmolt.so")
+_SOURCES = ["rows.cu", "lmhead_fwd.cu", "lmhead_bwd.cu", "api.cu"]
+ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+STATUS = {
+    0: "MOLT_OK", 1: "MOLT_ERR_INVALID_ARG", 2: "MOLT_ERR_UNSUPPORTED_SHAPE", 3: "MOLT_ERR_UNSORTED_GROUPS",
+    4: "MOLT_ERR_ZERO_DENOM", 5: "MOLT_ERR_CUDA", 6: "MOLT_ERR_DEVICE_TIMEOUT", 7: "MOLT_ERR_NO_MEMORY",
+    8: "MOLT_ERR_TOKEN_RANGE", 9: "MOLT_ERR_WORKSPACE",
+}
+DEV_FLAGS = {"timeout": 1, "token_range": 2, "zero_denom": 4, "unsorted_groups": 8}
+
+
+def lib_path() -> str:
+    return _LIB
+
+
+def _nvcc() -> str:
+    for c in (os.environ.get("NVCC"), "/usr/local/cuda/bin/nvcc", "nvcc"):
+        if c and (os.path.sep not in c or os.path.exists(c)):
+            return c
+    return "nvcc"
+
+
+def build(verbose: bool = False, force: bool = False) -> str:
+    """Compile the CUDA sources for sm_103a (in parallel) and link libmolt.so
+    into this package directory.  Returns the library path."""
+    os.makedirs(_BUILD, exist_ok=True)
+    srcs = [os.path.join(_CSRC, s) for s in _SOURCES]
+    deps = srcs + [os.path.join(_CSRC, h) for h in os.listdir(_CSRC) if h.endswith(".cuh")] + [
+        os.path.join(_INCLUDE, "molt.h")]
+    if (not force and os.path.exists(_LIB)
+            and os.path.getmtime(_LIB) >= max(os.path.getmtime(d) for d in deps)):
+        return _LIB
+    nvcc = _nvcc()
+    common = [nvcc, "-std=c++17", "-O3", "-lineinfo", *ARCH_FLAGS, "-Xcompiler", "-fPIC", "-I", _INCLUDE]
+
+    def compile_one(src):
+        obj = os.path.join(_BUILD, os.path.basename(src).replace(".cu", ".o"))
+        cmd = common + ["-c", src, "-o", obj]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed for {src}:\n{r.stdout}\n{r.stderr}")
+        if verbose:
+            sys.stdout.write(r.stdout + r.stderr)
+        return obj
+
+    with ThreadPoolExecutor(max_workers=len(srcs)) as ex:
+        objs = list(ex.map(compile_one, srcs))
+    tmp = _LIB + ".tmp"
+    cmd = [nvcc, "-shared", *ARCH_FLAGS, "-cudart", "shared", "-o", tmp, *objs,
+           "-Xlinker", "-rpath,/usr/local/cuda/lib64"]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+class MoltError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+_lib = None
+
+
+def load():
+    """Load libmolt.so (build() must have run).  Raises if it is missing."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB):
+        raise RuntimeError(f"{_LIB} is not built; call paper_2607_21653_gb300.build() first")
+    L = ctypes.CDLL(_LIB)
+    P, I64, I32, F, D, SZ = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_float, ctypes.c_double,
+                             ctypes.c_size_t)
+    sig = {
+        "molt_status_string": (ctypes.c_char_p, [I32]),
+        "molt_last_error": (ctypes.c_char_p, []),
+        "molt_version": (I32, []),
+        "molt_device_status": (I32, [P, ctypes.POINTER(ctypes.c_uint32)]),
+        "molt_group_advantages": (I32, [P, P, I64, D, P, P]),
+        "molt_broadcast_advantages": (I32, [P, P, I64, I64, P, P]),
+        "molt_mask_count": (I32, [P, I64, P, P]),
+        "molt_token_logprobs_workspace_bytes": (SZ, [I64, I64, I64]),
+        "molt_token_logprobs_fwd": (I32, [P, P, P, P, I64, I64, I64, P, P, P, SZ, P]),
+        "molt_policy_loss_workspace_bytes": (SZ, [I64, I64, I64]),
+        "molt_policy_loss_fwd_bwd": (I32, [P, P, P, P, P, P, I64, I64, I64, F, F, D, P, P, P, I32, P, P, P, P,
+                                            P, SZ, P]),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(L, name)
+        fn.restype = res
+        fn.argtypes = args
+    _lib = L
+    return L
+
+
+def header_functions() -> list[str]:
+    """Names of the functions declared in include/molt.h."""
+    with open(os.path.join(_INCLUDE, "molt.h")) as f:
+        txt = f.read()
+    return sorted(set(re.findall(r"\b(molt_[a-z0-9_]+)\s*\(", txt)))
+
+
+def _check(status: int):
+    if status != 0:
+        msg = load().molt_last_error().decode()
+        raise MoltError(status, msg)
+
+
+# ---------------------------------------------------------------- torch glue
+def _torch():
+    import torch
+    return torch
+
+
+def _ptr(t, dtype=None, name="tensor"):
+    """Device pointer of a contiguous CUDA tensor (None -> NULL)."""
+    if t is None:
+        return None
+    torch = _torch()
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def _stream(stream=None):
+    torch = _torch()
+    s = torch.cuda.current_stream() if stream is None else stream
+    return s.cuda_stream
+
+
+_ws_cache: dict = {}
+
+
+def _workspace(nbytes: int, device, key: str):
+    """Workspace buffer from the torch caching allocator, reused per (device, key)."""
+    torch = _torch()
+    k = (str(device), key)
+    buf = _ws_cache.get(k)
+    if buf is None or buf.numel() < nbytes:
+        buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+        _ws_cache[k] = buf
+    return buf
+
+
+def device_status(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the device status bits."""
+    flags = ctypes.c_uint32(0)
+    st = load().molt_device_status(_stream(stream), ctypes.byref(flags))
+    if st not in (0, 3, 4, 6, 8):
+        _check(st)
+    return int(flags.value)
+
+
+def group_advantages(rewards, group_ids, eps: float = 1e-6, out=None, stream=None):
+    torch = _torch()
+    n = rewards.shape[0]
+    out = torch.empty(n, dtype=torch.float32, device=rewards.device) if out is None else out
+    _check(load().molt_group_advantages(_ptr(rewards, torch.float32, "rewards"), _ptr(group_ids, torch.int32, "group_ids"),
+                                        n, float(eps), _ptr(out, torch.float32, "out"), _stream(stream)))
+    return out
+
+
+def broadcast_advantages(adv_resp, resp_of_token, out=None, stream=None):
+    torch = _torch()
+    T = resp_of_token.shape[0]
+    out = torch.empty(T, dtype=torch.float32, device=resp_of_token.device) if out is None else out
+    _check(load().molt_broadcast_advantages(_ptr(adv_resp, torch.float32, "adv_resp"),
+                                            _ptr(resp_of_token, torch.int32, "resp_of_token"), adv_resp.shape[0], T,
+                                            _ptr(out, torch.float32, "out"), _stream(stream)))
+    return out
+
+
+def mask_count(mask, out=None, stream=None):
+    torch = _torch()
+    out = torch.empty(1, dtype=torch.int64, device=mask.device) if out is None else out
+    _check(load().molt_mask_count(_ptr(mask, torch.uint8, "mask"), mask.shape[0], _ptr(out, torch.int64, "out"),
+                                  _stream(stream)))
+    return out
+
+
+def token_logprobs_workspace_bytes(T, H, V) -> int:
+    return int(load().molt_token_logprobs_workspace_bytes(T, H, V))
+
+
+def policy_loss_workspace_bytes(T, H, V) -> int:
+    return int(load().molt_policy_loss_workspace_bytes(T, H, V))
+
+
+def _bf16_bits(t, name):
+    torch = _torch()
+    if t.dtype == torch.bfloat16:
+        return _ptr(t, None, name)
+    if t.dtype in (torch.uint16, torch.int16):
+        return _ptr(t, None, name)
+    raise TypeError(f"{name} must be bfloat16 (or its 16-bit pattern)")
+
+
+def token_logprobs(hidden, weight, tokens, mask=None, want_entropy=True, stream=None, workspace=None):
+    """logp[T] and entropy[T] (fp32) of the generated tokens; rows with mask 0 give 0."""
+    torch = _torch()
+    T, H = hidden.shape
+    V = weight.shape[0]
+    logp = torch.empty(T, dtype=torch.float32, device=hidden.device)
+    ent = torch.empty(T, dtype=torch.float32, device=hidden.device) if want_entropy else None
+    nbytes = token_logprobs_workspace_bytes(T, H, V)
+    ws = workspace if workspace is not None else _workspace(nbytes, hidden.device, "logprobs")
+    _check(load().molt_token_logprobs_fwd(_bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"),
+                                          _ptr(tokens, torch.int32, "tokens"), _ptr(mask, torch.uint8, "mask"),
+                                          T, H, V, _ptr(logp), _ptr(ent), ws.data_ptr(), ws.numel(),
+                                          _stream(stream)))
+    return logp, ent
+
+
+def policy_loss_fwd_bwd(hidden, weight, tokens, behavior_logp, adv, mask=None, clip_lo=0.2, clip_hi=0.2,
+                        denom=0.0, dW=None, accumulate_dW=False, want_token_outputs=True, stream=None,
+                        workspace=None):
+    """Fused clipped-surrogate loss (Eq. 2 token-mean) forward + backward.
+
+    Returns dict(loss [1] fp32, dhidden [T,H] bf16, dW [V,H] fp32, logp, entropy,
+    token_loss [T] fp32 (None unless want_token_outputs), stats [8 x 8 bytes])."""
+    torch = _torch()
+    T, H = hidden.shape
+    V = weight.shape[0]
+    dev = hidden.device
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    dh = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
+    if dW is None:
+        dW = torch.empty(V, H, dtype=torch.float32, device=dev)
+        accumulate_dW = False
+    stats = torch.zeros(8, dtype=torch.float64, device=dev)
+    logp = ent = tl = None
+    if want_token_outputs:
+        logp = torch.empty(T, dtype=torch.float32, device=dev)
+        ent = torch.empty(T, dtype=torch.float32, device=dev)
+        tl = torch.empty(T, dtype=torch.float32, device=dev)
+    nbytes = policy_loss_workspace_bytes(T, H, V)
+    ws = workspace if workspace is not None else _workspace(nbytes, dev, "policy_loss")
+    _check(load().molt_policy_loss_fwd_bwd(
+        _bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"), _ptr(tokens, torch.int32, "tokens"),
+        _ptr(behavior_logp, torch.float32, "behavior_logp"), _ptr(adv, torch.float32, "adv"),
+        _ptr(mask, torch.uint8, "mask"), T, H, V, float(clip_lo), float(clip_hi), float(denom), _ptr(loss),
+        _ptr(dh), _ptr(dW, torch.float32, "dW"), 1 if accumulate_dW else 0, _ptr(logp), _ptr(ent), _ptr(tl),
+        _ptr(stats), ws.data_ptr(), ws.numel(), _stream(stream)))
+    return {"loss": loss, "dhidden": dh, "dW": dW, "logp": logp, "entropy": ent, "token_loss": tl,
+            "stats": stats}
+
+
+def stats_dict(stats_tensor) -> dict:
+    """Decode the molt_stats struct (5 doubles + 3 int64) copied to the host."""
+    import numpy as np
+    raw = stats_tensor.detach().cpu().numpy().view(np.uint8).tobytes()
+    d = np.frombuffer(raw[:40], dtype=np.float64)
+    i = np.frombuffer(raw[40:64], dtype=np.int64)
+    return {"denom": float(d[0]), "loss": float(d[1]), "sum_ratio": float(d[2]), "sum_entropy": float(d[3]),
+            "max_abs_log_ratio": float(d[4]), "n_active": int(i[0]), "n_clip_low": int(i[1]),
+            "n_clip_high": int(i[2])}

@@ -1,0 +1,432 @@
+// C ABI of the library (include/molt.h): argument validation, workspace
+// layout, TMA tensor maps and the launch sequence of each entry point.
+#include <atomic>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+#include <string>
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include "../../include/molt.h"
+#include "molt_internal.cuh"
+#include "ptx.cuh"
+
+// Per-device status word set by the kernels (MOLT_DEV_* bits).
+__device__ unsigned g_molt_status_word;
+
+namespace molt {
+namespace {
+
+thread_local std::string t_last_error;
+
+molt_status fail(molt_status s, const std::string& msg) {
+  t_last_error = msg;
+  return s;
+}
+molt_status cuda_fail(cudaError_t e, const char* what) {
+  t_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+  return MOLT_ERR_CUDA;
+}
+
+constexpr int kMaxDevices = 64;
+struct DeviceInfo {
+  std::once_flag once;
+  int n_sm = 0;
+  unsigned* status = nullptr;
+  cudaError_t err = cudaSuccess;
+};
+DeviceInfo g_dev[kMaxDevices];
+
+// SM count and the address of the status word on the current device
+const DeviceInfo* device_info(molt_status* st) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    *st = cuda_fail(e, "cudaGetDevice");
+    return nullptr;
+  }
+  if (dev < 0 || dev >= kMaxDevices) {
+    *st = fail(MOLT_ERR_CUDA, "device ordinal out of range");
+    return nullptr;
+  }
+  DeviceInfo& d = g_dev[dev];
+  std::call_once(d.once, [&d, dev]() {
+    d.err = cudaDeviceGetAttribute(&d.n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (d.err == cudaSuccess) d.err = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.status), g_molt_status_word);
+  });
+  if (d.err != cudaSuccess) {
+    *st = cuda_fail(d.err, "device query");
+    return nullptr;
+  }
+  *st = MOLT_OK;
+  return &d;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static std::once_flag once;
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  std::call_once(once, []() {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D row-major tensor map: `rows` x `cols` elements, box `box_cols` x `box_rows`
+molt_status make_tmap(CUtensorMap* m, CUtensorMapDataType dt, int elem_bytes, const void* base, uint64_t rows,
+                      uint64_t cols, uint32_t box_cols, uint32_t box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return fail(MOLT_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * static_cast<uint64_t>(elem_bytes)};
+  cuuint32_t box[2] = {box_cols, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(MOLT_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
+  return MOLT_OK;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline size_t up256(size_t x) { return (x + 255) & ~size_t(255); }
+
+int64_t round_tiles(int64_t T) { return ((T + kTileM - 1) / kTileM) * kTileM; }
+
+// vocab splits of the forward pass: enough units for ~16 waves of CTAs when
+// every row is active, never more splits than vocab tiles
+int choose_splits(int64_t Tcap, int64_t V, int n_sm) {
+  const int64_t n_vt = (V + kFwdBN - 1) / kFwdBN;
+  const int64_t n_mt = Tcap / kTileM;
+  int64_t S = (16 * static_cast<int64_t>(n_sm) + n_mt - 1) / n_mt;
+  if (S < 1) S = 1;
+  if (S > n_vt) S = n_vt;
+  return static_cast<int>(S);
+}
+
+struct Layout {
+  size_t counts, row_map, pos, tok_p, b_p, adv_p, h_p, part, zx, lse, coef, tile_flag, tile_list, red, dh32, total;
+};
+
+Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd) {
+  const int64_t Tcap = round_tiles(T);
+  const int64_t ntile = Tcap / kTileM;
+  Layout L{};
+  size_t o = 0;
+  auto take = [&o](size_t bytes) {
+    size_t r = o;
+    o += up256(bytes);
+    return r;
+  };
+  L.counts = take(64);
+  L.row_map = take(T * 4);
+  L.pos = take(T * 4);
+  L.tok_p = take(Tcap * 4);
+  L.b_p = take(Tcap * 4);
+  L.adv_p = take(Tcap * 4);
+  L.h_p = take(Tcap * H * 2);
+  L.part = take(static_cast<size_t>(S) * Tcap * 16);
+  L.zx = take(Tcap * 4);
+  L.lse = take(Tcap * 4);
+  L.coef = take(Tcap * 4);
+  L.tile_flag = take(ntile * 4);
+  L.tile_list = take(ntile * 4);
+  L.red = take(ntile * kRedSlots * 8);
+  L.dh32 = with_bwd ? take(Tcap * H * 4) : o;
+  L.total = o + 256;   // slack for aligning the caller's base pointer
+  (void)V;
+  return L;
+}
+
+Workspace carve(void* base, const Layout& L) {
+  uint8_t* p = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(base) + 255) & ~uintptr_t(255));
+  Workspace w{};
+  w.counts = reinterpret_cast<int32_t*>(p + L.counts);
+  w.row_map = reinterpret_cast<int32_t*>(p + L.row_map);
+  w.pos_of_row = reinterpret_cast<int32_t*>(p + L.pos);
+  w.tok_p = reinterpret_cast<int32_t*>(p + L.tok_p);
+  w.b_p = reinterpret_cast<float*>(p + L.b_p);
+  w.adv_p = reinterpret_cast<float*>(p + L.adv_p);
+  w.h_p = reinterpret_cast<uint16_t*>(p + L.h_p);
+  w.part = reinterpret_cast<float4*>(p + L.part);
+  w.zx = reinterpret_cast<float*>(p + L.zx);
+  w.lse = reinterpret_cast<float*>(p + L.lse);
+  w.coef = reinterpret_cast<float*>(p + L.coef);
+  w.tile_flag = reinterpret_cast<int32_t*>(p + L.tile_flag);
+  w.tile_list = reinterpret_cast<int32_t*>(p + L.tile_list);
+  w.red = reinterpret_cast<double*>(p + L.red);
+  w.dh32 = reinterpret_cast<float*>(p + L.dh32);
+  return w;
+}
+
+molt_status check_shape(int64_t T, int64_t H, int64_t V) {
+  if (T < 0 || V < 1 || H < 1) return fail(MOLT_ERR_INVALID_ARG, "sizes must satisfy T >= 0, H >= 1, V >= 1");
+  if (H % 64 != 0) return fail(MOLT_ERR_UNSUPPORTED_SHAPE, "H must be a multiple of 64");
+  if (T >= (int64_t(1) << 31) - kTileM || V >= (int64_t(1) << 31) || H > 65536)
+    return fail(MOLT_ERR_UNSUPPORTED_SHAPE, "T and V must be below 2^31 and H at most 65536");
+  return MOLT_OK;
+}
+
+// Scratch memory of one call: the caller's buffer, or a stream-ordered allocation.
+struct Scratch {
+  void* ptr = nullptr;
+  bool owned = false;
+  cudaStream_t s = nullptr;
+  ~Scratch() {
+    if (owned && ptr) cudaFreeAsync(ptr, s);
+  }
+};
+
+molt_status get_scratch(Scratch& sc, void* ws, size_t ws_bytes, size_t need, cudaStream_t s) {
+  sc.s = s;
+  if (ws) {
+    if (ws_bytes < need)
+      return fail(MOLT_ERR_WORKSPACE, "workspace of " + std::to_string(ws_bytes) + " bytes, need " +
+                                          std::to_string(need));
+    sc.ptr = ws;
+    return MOLT_OK;
+  }
+  cudaError_t e = cudaMallocAsync(&sc.ptr, need, s);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    sc.ptr = nullptr;
+    return fail(MOLT_ERR_NO_MEMORY, std::string("cudaMallocAsync: ") + cudaGetErrorString(e));
+  }
+  sc.owned = true;
+  return MOLT_OK;
+}
+
+#define MOLT_CUDA(call, what)                        \
+  do {                                               \
+    cudaError_t e_ = (call);                         \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+#define MOLT_TRY(call)                   \
+  do {                                   \
+    molt_status s_ = (call);             \
+    if (s_ != MOLT_OK) return s_;        \
+  } while (0)
+
+// Shared front half of both LM-head calls: compaction, packed gather and the
+// forward kernel (tensor maps already encoded by the caller).
+molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int32_t* tokens, const uint8_t* mask,
+                        const float* b, const float* adv, int64_t T, int64_t H, int64_t V, int S,
+                        const Workspace& w, const CUtensorMap& tm_h, const CUtensorMap& tm_w, cudaStream_t s) {
+  const int64_t Tcap = round_tiles(T);
+  MOLT_CUDA(launch_compact(mask, static_cast<int>(T), w, s), "compact");
+  MOLT_CUDA(launch_gather(hidden, tokens, b, adv, static_cast<int>(T), static_cast<int>(Tcap), static_cast<int>(H),
+                          w, di->n_sm, s),
+            "gather");
+  FwdArgs fa{};
+  fa.tok_p = w.tok_p;
+  fa.counts = w.counts;
+  fa.rows_cap = static_cast<int>(Tcap);
+  fa.V = static_cast<int>(V);
+  fa.H = static_cast<int>(H);
+  fa.n_split = S;
+  fa.n_vtiles = static_cast<int>((V + kFwdBN - 1) / kFwdBN);
+  fa.part = w.part;
+  fa.zx = w.zx;
+  fa.err = di->status;
+  MOLT_CUDA(launch_lmhead_fwd(tm_h, tm_w, fa, di->n_sm, s), "lmhead forward");
+  return MOLT_OK;
+}
+
+}  // namespace
+}  // namespace molt
+
+using namespace molt;
+
+extern "C" {
+
+const char* molt_status_string(molt_status s) {
+  switch (s) {
+    case MOLT_OK: return "ok";
+    case MOLT_ERR_INVALID_ARG: return "invalid argument";
+    case MOLT_ERR_UNSUPPORTED_SHAPE: return "unsupported shape";
+    case MOLT_ERR_UNSORTED_GROUPS: return "group ids are not sorted";
+    case MOLT_ERR_ZERO_DENOM: return "zero token-mean denominator";
+    case MOLT_ERR_CUDA: return "CUDA error";
+    case MOLT_ERR_DEVICE_TIMEOUT: return "device pipeline wait timed out";
+    case MOLT_ERR_NO_MEMORY: return "out of device memory";
+    case MOLT_ERR_TOKEN_RANGE: return "token id out of range";
+    case MOLT_ERR_WORKSPACE: return "workspace too small";
+  }
+  return "unknown status";
+}
+
+const char* molt_last_error(void) { return t_last_error.c_str(); }
+
+int molt_version(void) { return 1; }
+
+molt_status molt_device_status(cudaStream_t stream, uint32_t* flags) {
+  if (!flags) return fail(MOLT_ERR_INVALID_ARG, "flags is NULL");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  MOLT_CUDA(cudaStreamSynchronize(stream), "cudaStreamSynchronize");
+  unsigned v = 0;
+  MOLT_CUDA(cudaMemcpy(&v, di->status, sizeof(v), cudaMemcpyDeviceToHost), "read status word");
+  MOLT_CUDA(cudaMemset(di->status, 0, sizeof(unsigned)), "clear status word");
+  *flags = v;
+  if (v & MOLT_DEV_TIMEOUT) return fail(MOLT_ERR_DEVICE_TIMEOUT, "a pipeline wait timed out");
+  if (v & MOLT_DEV_TOKEN_RANGE) return fail(MOLT_ERR_TOKEN_RANGE, "a token id on an active row is outside [0, V)");
+  if (v & MOLT_DEV_ZERO_DENOM) return fail(MOLT_ERR_ZERO_DENOM, "no active token and no window denominator");
+  if (v & MOLT_DEV_UNSORTED_GROUPS) return fail(MOLT_ERR_UNSORTED_GROUPS, "group ids decrease somewhere");
+  return MOLT_OK;
+}
+
+molt_status molt_group_advantages(const float* rewards, const int32_t* group_ids, int64_t n_resp, double eps,
+                                  float* adv_out, cudaStream_t stream) {
+  if (n_resp < 0 || n_resp >= (int64_t(1) << 26)) return fail(MOLT_ERR_INVALID_ARG, "n_resp out of range");
+  if (n_resp == 0) return MOLT_OK;
+  if (!rewards || !group_ids || !adv_out) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (!(eps >= 0.0) || eps != eps) return fail(MOLT_ERR_INVALID_ARG, "eps must be >= 0");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  MOLT_CUDA(launch_group_advantages(rewards, group_ids, static_cast<int>(n_resp), eps, adv_out, di->status, stream),
+            "group advantages");
+  return MOLT_OK;
+}
+
+molt_status molt_broadcast_advantages(const float* adv_resp, const int32_t* resp_of_token, int64_t n_resp,
+                                      int64_t T, float* adv_tok, cudaStream_t stream) {
+  if (T < 0 || n_resp < 0 || T >= (int64_t(1) << 31) || n_resp >= (int64_t(1) << 31))
+    return fail(MOLT_ERR_INVALID_ARG, "sizes out of range");
+  if (T == 0) return MOLT_OK;
+  if (!adv_resp || !resp_of_token || !adv_tok) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  MOLT_CUDA(launch_broadcast(adv_resp, resp_of_token, static_cast<int>(n_resp), static_cast<int>(T), adv_tok, stream),
+            "broadcast");
+  return MOLT_OK;
+}
+
+molt_status molt_mask_count(const uint8_t* mask, int64_t T, int64_t* count_out, cudaStream_t stream) {
+  if (T < 0) return fail(MOLT_ERR_INVALID_ARG, "T < 0");
+  if (!count_out || (T > 0 && !mask)) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (T > 0 && !aligned16(mask)) return fail(MOLT_ERR_INVALID_ARG, "mask must be 16-byte aligned");
+  if ((reinterpret_cast<uintptr_t>(count_out) & 7u) != 0) return fail(MOLT_ERR_INVALID_ARG, "count_out misaligned");
+  MOLT_CUDA(launch_mask_count(mask, T, count_out, stream), "mask count");
+  return MOLT_OK;
+}
+
+size_t molt_token_logprobs_workspace_bytes(int64_t T, int64_t H, int64_t V) {
+  if (check_shape(T, H, V) != MOLT_OK) return 0;
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  const int n_sm = di ? di->n_sm : 152;
+  const int64_t Tcap = round_tiles(T);
+  return layout(T, H, V, choose_splits(Tcap > 0 ? Tcap : kTileM, V, n_sm), false).total;
+}
+
+size_t molt_policy_loss_workspace_bytes(int64_t T, int64_t H, int64_t V) {
+  if (check_shape(T, H, V) != MOLT_OK) return 0;
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  const int n_sm = di ? di->n_sm : 152;
+  const int64_t Tcap = round_tiles(T);
+  return layout(T, H, V, choose_splits(Tcap > 0 ? Tcap : kTileM, V, n_sm), true).total;
+}
+
+molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                                    const uint8_t* mask, int64_t T, int64_t H, int64_t V, float* logp_out,
+                                    float* entropy_out, void* workspace, size_t workspace_bytes,
+                                    cudaStream_t stream) {
+  MOLT_TRY(check_shape(T, H, V));
+  if (T == 0) return MOLT_OK;
+  if (!hidden || !W || !tokens || !logp_out) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(hidden) || !aligned16(W)) return fail(MOLT_ERR_INVALID_ARG, "hidden and W must be 16-byte aligned");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  const int64_t Tcap = round_tiles(T);
+  const int S = choose_splits(Tcap, V, di->n_sm);
+  const Layout L = layout(T, H, V, S, false);
+  Scratch sc;
+  MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
+  const Workspace w = carve(sc.ptr, L);
+  CUtensorMap tm_h, tm_w;
+  MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
+  MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
+  MOLT_TRY(run_forward(di, hidden, tokens, mask, nullptr, nullptr, T, H, V, S, w, tm_h, tm_w, stream));
+  MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
+  if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
+  MOLT_CUDA(launch_merge(false, static_cast<int>(Tcap), static_cast<int>(V), S, 0.0, 0.f, 0.f, w, logp_out,
+                         entropy_out, nullptr, di->status, stream),
+            "merge");
+  return MOLT_OK;
+}
+
+molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                                     const float* behavior_logp, const float* adv, const uint8_t* mask,
+                                     int64_t T, int64_t H, int64_t V, float clip_lo, float clip_hi,
+                                     double denom, float* loss_out, uint16_t* dhidden_out, float* dW_out,
+                                     int accumulate_dW, float* logp_out, float* entropy_out,
+                                     float* token_loss_out, molt_stats* stats_out, void* workspace,
+                                     size_t workspace_bytes, cudaStream_t stream) {
+  MOLT_TRY(check_shape(T, H, V));
+  if (!hidden || !W || !tokens || !behavior_logp || !adv || !loss_out || !dhidden_out || !dW_out)
+    return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(hidden) || !aligned16(W) || !aligned16(dhidden_out) || !aligned16(dW_out))
+    return fail(MOLT_ERR_INVALID_ARG, "hidden, W, dhidden and dW must be 16-byte aligned");
+  if (!(clip_lo >= 0.f && clip_lo < 1.f) || !(clip_hi >= 0.f) || clip_hi != clip_hi || clip_hi > 1e30f)
+    return fail(MOLT_ERR_INVALID_ARG, "clip bounds must satisfy 0 <= clip_lo < 1 and clip_hi >= 0");
+  if (denom != denom) return fail(MOLT_ERR_INVALID_ARG, "denom is NaN");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  if (T == 0) {
+    // nothing to compute: loss 0, stats zero, dW untouched or zeroed
+    MOLT_CUDA(cudaMemsetAsync(loss_out, 0, sizeof(float), stream), "memset loss");
+    if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, V * H * sizeof(float), stream), "memset dW");
+    if (stats_out) MOLT_CUDA(cudaMemsetAsync(stats_out, 0, sizeof(molt_stats), stream), "memset stats");
+    return MOLT_OK;
+  }
+  const int64_t Tcap = round_tiles(T);
+  const int S = choose_splits(Tcap, V, di->n_sm);
+  const Layout L = layout(T, H, V, S, true);
+  Scratch sc;
+  MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
+  const Workspace w = carve(sc.ptr, L);
+  CUtensorMap tm_h, tm_w, tm_wz, tm_wn, tm_dh, tm_dw;
+  MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
+  MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
+  MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kBwdBV));
+  MOLT_TRY(make_tmap(&tm_wn, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, 64));
+  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
+  MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
+  MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
+  if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
+  if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
+  if (token_loss_out) MOLT_CUDA(cudaMemsetAsync(token_loss_out, 0, T * sizeof(float), stream), "memset token loss");
+  MOLT_CUDA(launch_merge(true, static_cast<int>(Tcap), static_cast<int>(V), S, denom, clip_lo, clip_hi, w, logp_out,
+                         entropy_out, token_loss_out, di->status, stream),
+            "merge");
+  MOLT_CUDA(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, di->status, stream), "finalize");
+  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
+  if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
+  BwdArgs ba{};
+  ba.tok_p = w.tok_p;
+  ba.lse = w.lse;
+  ba.coef = w.coef;
+  ba.counts = w.counts;
+  ba.tile_list = w.tile_list;
+  ba.V = static_cast<int>(V);
+  ba.H = static_cast<int>(H);
+  ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
+  ba.tile_group = 16;
+  ba.err = di->status;
+  MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
+  return MOLT_OK;
+}
+
+}  // extern "C"

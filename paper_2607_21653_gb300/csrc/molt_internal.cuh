@@ -1,0 +1,82 @@
+// Internal launch interface between the C-ABI layer (api.cu) and the kernels.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+namespace molt {
+
+constexpr int kTileM = 128;   // token rows per tile (TMEM lanes)
+constexpr int kFwdBN = 256;   // vocab columns per forward MMA tile
+constexpr int kBwdBV = 256;   // vocab columns per backward unit
+constexpr int kBK = 64;       // K elements per 128-byte swizzled row
+
+// Device pointers into one call's workspace (all regions 256-byte aligned).
+struct Workspace {
+  int32_t* counts;      // [0] active rows n, [1] active backward tiles
+  int32_t* row_map;     // [T]    packed row -> original row
+  int32_t* pos_of_row;  // [T]    original row -> packed row or -1
+  int32_t* tok_p;       // [Tcap] packed tokens
+  float* b_p;           // [Tcap] packed behaviour log-probs
+  float* adv_p;         // [Tcap] packed advantages
+  uint16_t* h_p;        // [Tcap, H] packed hidden rows (bf16 bits), rows >= n zeroed
+  float4* part;         // [S, Tcap] per-split (max, sum exp, sum exp*(z-max), -)
+  float* zx;            // [Tcap] target logit
+  float* lse;           // [Tcap]
+  float* coef;          // [Tcap] m c / D
+  int32_t* tile_flag;   // [Tcap/128]
+  int32_t* tile_list;   // [Tcap/128]
+  double* red;          // [n_tiles * kRedSlots] per-tile partial sums
+  float* dh32;          // [Tcap, H] fp32 dhidden accumulator (loss call only)
+};
+constexpr int kRedSlots = 8;
+
+struct FwdArgs {
+  const int32_t* tok_p;
+  const int32_t* counts;
+  int rows_cap;
+  int V, H;
+  int n_split;
+  int n_vtiles;
+  float4* part;
+  float* zx;
+  unsigned* err;
+};
+
+struct BwdArgs {
+  const int32_t* tok_p;
+  const float* lse;
+  const float* coef;
+  const int32_t* counts;     // counts[1] = active tiles
+  const int32_t* tile_list;
+  int V, H;
+  int n_vchunks;
+  int tile_group;            // token tiles per raster group
+  unsigned* err;
+};
+
+// rows.cu
+cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
+                                    unsigned* err, cudaStream_t s);
+cudaError_t launch_broadcast(const float* adv, const int32_t* rot, int n_resp, int T, float* out, cudaStream_t s);
+cudaError_t launch_mask_count(const uint8_t* mask, int64_t T, int64_t* out, cudaStream_t s);
+cudaError_t launch_compact(const uint8_t* mask, int T, const Workspace& ws, cudaStream_t s);
+cudaError_t launch_gather(const uint16_t* hidden, const int32_t* tokens, const float* b, const float* adv, int T,
+                          int Tcap, int H, const Workspace& ws, int n_sm, cudaStream_t s);
+cudaError_t launch_merge(bool loss_mode, int Tcap, int V, int n_split, double denom, float clip_lo, float clip_hi,
+                         const Workspace& ws, float* logp_out, float* ent_out, float* tokloss_out, unsigned* err,
+                         cudaStream_t s);
+cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* loss_out, void* stats_out,
+                            unsigned* err, cudaStream_t s);
+cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s);
+
+// lmhead_fwd.cu
+cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,
+                              cudaStream_t s);
+// lmhead_bwd.cu
+cudaError_t launch_lmhead_bwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w_z, const CUtensorMap& tm_w_n,
+                              const CUtensorMap& tm_dh, const CUtensorMap& tm_dw, const BwdArgs& a, int grid,
+                              cudaStream_t s);
+
+}  // namespace molt

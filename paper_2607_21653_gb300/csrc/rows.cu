@@ -1,0 +1,472 @@
+// Row-level kernels of the policy-update path: GRPO advantages, advantage
+// broadcast, mask count, active-row compaction, packed gathers, the split-vocab
+// merge with the clipped surrogate, the fixed-order loss reduction and the
+// dhidden cast.  None of these is a contraction; they are launch- or HBM-bound.
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "molt_internal.cuh"
+#include "ptx.cuh"
+
+namespace molt {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+// ---------------------------------------------------------------------------
+// GRPO advantages (Sec. 4.5 estimator list; Sec. 4.2 one reward per rollout).
+// One warp per response index; the warp whose index starts a run of equal ids
+// processes that group.  Lanes load the rewards coalesced, 32 at a time, and
+// lane 0 folds them with shuffles in index order, so the fp64 sums run in the
+// same order as a sequential loop.  Explicit _rn intrinsics keep the compiler
+// from contracting a multiply and an add into an FMA.
+// ---------------------------------------------------------------------------
+__global__ void group_adv_kernel(const float* __restrict__ r, const int32_t* __restrict__ gid, int n, double eps,
+                                 float* __restrict__ out, unsigned* err) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (warp >= n) return;
+  const int start = warp;
+  const int g = gid[start];
+  if (start > 0) {
+    const int gp = gid[start - 1];
+    if (gp == g) return;
+    if (gp > g && lane == 0) atomicOr(err, kDevErrUnsortedGroups);
+  }
+  // end of the run
+  int end = start;
+  for (int base = start;; base += 32) {
+    const int j = base + lane;
+    const bool same = (j < n) && (gid[j] == g);
+    const unsigned m = __ballot_sync(0xffffffffu, same);
+    if (m == 0xffffffffu) {
+      end = base + 32;
+      continue;
+    }
+    end = base + __ffs(~m) - 1;
+    break;
+  }
+  const int cnt = end - start;
+  if (cnt == 1) {
+    if (lane == 0) out[start] = 0.0f;
+    return;
+  }
+  double s = 0.0;
+  for (int base = start; base < end; base += 32) {
+    const int j = base + lane;
+    const double v = (j < end) ? static_cast<double>(r[j]) : 0.0;
+    const int k = min(32, end - base);
+    for (int i = 0; i < k; ++i) {
+      const double vi = __shfl_sync(0xffffffffu, v, i);
+      s = __dadd_rn(s, vi);
+    }
+  }
+  const double mean = __ddiv_rn(__shfl_sync(0xffffffffu, s, 0), static_cast<double>(cnt));
+  double ss = 0.0;
+  for (int base = start; base < end; base += 32) {
+    const int j = base + lane;
+    const double d = (j < end) ? __dsub_rn(static_cast<double>(r[j]), mean) : 0.0;
+    const double d2 = __dmul_rn(d, d);
+    const int k = min(32, end - base);
+    for (int i = 0; i < k; ++i) ss = __dadd_rn(ss, __shfl_sync(0xffffffffu, d2, i));
+  }
+  ss = __shfl_sync(0xffffffffu, ss, 0);
+  const double sd = __dsqrt_rn(__ddiv_rn(ss, static_cast<double>(cnt - 1)));
+  const double den = __dadd_rn(sd, eps);
+  for (int base = start; base < end; base += 32) {
+    const int j = base + lane;
+    if (j < end) {
+      const double d = __dsub_rn(static_cast<double>(r[j]), mean);
+      out[j] = __double2float_rn(__ddiv_rn(d, den));
+    }
+  }
+}
+
+__global__ void broadcast_kernel(const float* __restrict__ adv, const int32_t* __restrict__ rot, int n_resp, int T,
+                                 float* __restrict__ out) {
+  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < T; t += gridDim.x * blockDim.x) {
+    const int k = rot[t];
+    out[t] = (k >= 0 && k < n_resp) ? adv[k] : 0.0f;
+  }
+}
+
+// sum of a uint8 mask: 16 bytes per load, per-block total, one atomic per block
+__global__ void mask_count_kernel(const uint8_t* __restrict__ mask, int64_t T,
+                                  unsigned long long* __restrict__ out) {
+  unsigned long long c = 0;
+  const int64_t nvec = T / 16;
+  const uint4* m4 = reinterpret_cast<const uint4*>(mask);
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < nvec; i += (int64_t)gridDim.x * blockDim.x) {
+    const uint4 v = m4[i];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) c += (w[q] & 0xFFu ? 1 : 0) + (w[q] & 0xFF00u ? 1 : 0) +
+                                     (w[q] & 0xFF0000u ? 1 : 0) + (w[q] & 0xFF000000u ? 1 : 0);
+  }
+  for (int64_t i = nvec * 16 + blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < T;
+       i += (int64_t)gridDim.x * blockDim.x)
+    c += mask[i] ? 1 : 0;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) c += __shfl_xor_sync(0xffffffffu, c, o);
+  __shared__ unsigned long long sh[32];
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = c;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long tot = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += sh[w];
+    if (tot) atomicAdd(out, tot);
+  }
+}
+
+// block-wide exclusive scan of one int per thread (blockDim.x = 1024)
+__device__ int block_exclusive_scan(int v, int* total) {
+  __shared__ int wsum[32];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) wsum[w] = x;
+  __syncthreads();
+  if (w == 0) {
+    int s = (lane < (int)(blockDim.x >> 5)) ? wsum[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, s, o);
+      if (lane >= o) s += y;
+    }
+    wsum[lane] = s;
+  }
+  __syncthreads();
+  const int before = (w > 0 ? wsum[w - 1] : 0) + x - v;
+  if (total) *total = wsum[(blockDim.x >> 5) - 1];
+  __syncthreads();
+  return before;
+}
+
+// order-preserving list of active rows (mask != 0): one block, each thread a
+// contiguous chunk
+__global__ void __launch_bounds__(1024) compact_kernel(const uint8_t* __restrict__ mask, int T,
+                                                       int32_t* __restrict__ row_map, int32_t* __restrict__ pos,
+                                                       int32_t* __restrict__ counts) {
+  const int per = (T + blockDim.x - 1) / blockDim.x;
+  const int b = threadIdx.x * per, e = min(T, b + per);
+  int c = 0;
+  for (int t = b; t < e; ++t) c += (mask == nullptr || mask[t]) ? 1 : 0;
+  int total;
+  int k = block_exclusive_scan(c, &total);
+  for (int t = b; t < e; ++t) {
+    if (mask == nullptr || mask[t]) {
+      row_map[k] = t;
+      pos[t] = k++;
+    } else {
+      pos[t] = -1;
+    }
+  }
+  if (threadIdx.x == 0) {
+    counts[0] = total;
+    counts[1] = 0;
+  }
+}
+
+// packed copies of the active rows; rows in [n, round_up(n,128)) are zeroed so
+// that the last tile holds finite values
+__global__ void gather_kernel(const uint16_t* __restrict__ hidden, const int32_t* __restrict__ tokens,
+                              const float* __restrict__ b, const float* __restrict__ adv, int Tcap, int H,
+                              const int32_t* __restrict__ row_map, const int32_t* __restrict__ counts,
+                              uint16_t* __restrict__ h_p, int32_t* __restrict__ tok_p, float* __restrict__ b_p,
+                              float* __restrict__ adv_p) {
+  const int n = counts[0];
+  const int nz = min(Tcap, ((n + kTileM - 1) / kTileM) * kTileM);
+  const int vpr = H / 8;   // 16-byte vectors per row
+  const int64_t total = (int64_t)nz * vpr;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int k = (int)(i / vpr), v = (int)(i - (int64_t)k * vpr);
+    uint4 val = make_uint4(0, 0, 0, 0);
+    if (k < n) {
+      const int t = row_map[k];
+      val = reinterpret_cast<const uint4*>(hidden + (int64_t)t * H)[v];
+      if (v == 0) {
+        tok_p[k] = tokens[t];
+        if (b_p) b_p[k] = b[t];
+        if (adv_p) adv_p[k] = adv[t];
+      }
+    } else if (v == 0) {
+      tok_p[k] = 0;
+      if (b_p) b_p[k] = 0.f;
+      if (adv_p) adv_p[k] = 0.f;
+    }
+    reinterpret_cast<uint4*>(h_p + (int64_t)k * H)[v] = val;
+  }
+}
+
+// deterministic 128-thread block sum (fixed tree)
+template <typename T>
+__device__ T block128_sum(T v, T* sh) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
+  __syncthreads();
+  T r = (sh[0] + sh[1]) + (sh[2] + sh[3]);
+  __syncthreads();
+  return r;
+}
+__device__ double block128_max(double v, double* sh) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmax(v, __shfl_xor_sync(0xffffffffu, v, o));
+  if ((threadIdx.x & 31) == 0) sh[threadIdx.x >> 5] = v;
+  __syncthreads();
+  double r = fmax(fmax(sh[0], sh[1]), fmax(sh[2], sh[3]));
+  __syncthreads();
+  return r;
+}
+
+// One block of 128 threads per packed tile: merge the per-split online
+// softmax partials of each row into lse, logp and entropy; in loss mode also
+// the ratio, the clipped surrogate (Sec. 4.5, PPO form), the Eq. 2 coefficient
+// m c / D, per-tile partial sums and the tile's activity flag.
+__global__ void __launch_bounds__(128) merge_kernel(
+    int loss_mode, int Tcap, int V, int n_split, double denom, float clip_lo, float clip_hi,
+    const int32_t* __restrict__ counts, const int32_t* __restrict__ row_map, const int32_t* __restrict__ tok_p,
+    const float* __restrict__ b_p, const float* __restrict__ adv_p, const float4* __restrict__ part,
+    const float* __restrict__ zx, float* __restrict__ lse_o, float* __restrict__ coef_o,
+    int32_t* __restrict__ tile_flag, double* __restrict__ red, float* __restrict__ logp_out,
+    float* __restrict__ ent_out, float* __restrict__ tokloss_out, unsigned* err) {
+  __shared__ double shd[4];
+  __shared__ long long shl[4];
+  const int n = counts[0];
+  const int n_tiles = (n + kTileM - 1) / kTileM;
+  if ((int)blockIdx.x >= n_tiles) return;
+  const int k = blockIdx.x * kTileM + threadIdx.x;
+  const bool act = k < n;
+  const double D = denom > 0.0 ? denom : static_cast<double>(n);
+  float logp = 0.f, ent = 0.f, coef = 0.f, tl = 0.f, ratio = 0.f;
+  int clip_lo_hit = 0, clip_hi_hit = 0;
+  double alr = 0.0;
+  if (act) {
+    float M = -INFINITY;
+    for (int s = 0; s < n_split; ++s) M = fmaxf(M, part[(int64_t)s * Tcap + k].x);
+    float S = 0.f, Q = 0.f;
+    for (int s = 0; s < n_split; ++s) {
+      const float4 p = part[(int64_t)s * Tcap + k];
+      if (p.y > 0.f) {
+        const float d = p.x - M;
+        const float f = ex2_approx(d * kLog2e);
+        S += f * p.y;
+        Q += f * (p.z + d * p.y);
+      }
+    }
+    const float logS = logf(S);
+    const float lse = M + logS;
+    const int x = tok_p[k];
+    if (x < 0 || x >= V) atomicOr(err, kDevErrTokenRange);
+    logp = zx[k] - lse;
+    ent = logS - Q / S;
+    lse_o[k] = lse;
+    if (loss_mode) {
+      const float b = b_p[k], A = adv_p[k];
+      ratio = expf(logp - b);
+      const float lo = 1.0f - clip_lo, hi = 1.0f + clip_hi;
+      const bool clipped = (A > 0.f && ratio > hi) || (A < 0.f && ratio < lo);
+      const float rc = fminf(fmaxf(ratio, lo), hi);
+      tl = clipped ? -(rc * A) : -(ratio * A);
+      const float c = clipped ? 0.f : ratio * A;
+      coef = (D > 0.0) ? static_cast<float>(static_cast<double>(c) / D) : 0.f;
+      clip_lo_hit = (clipped && A < 0.f) ? 1 : 0;
+      clip_hi_hit = (clipped && A > 0.f) ? 1 : 0;
+      alr = fabs(static_cast<double>(logp) - static_cast<double>(b));
+    }
+    const int t = row_map[k];
+    if (logp_out) logp_out[t] = logp;
+    if (ent_out) ent_out[t] = ent;
+    if (tokloss_out) tokloss_out[t] = tl;
+  }
+  if (!loss_mode) return;
+  if (k < Tcap) coef_o[k] = coef;
+  const int any = __syncthreads_or(coef != 0.f);
+  double* r = red + (int64_t)blockIdx.x * kRedSlots;
+  const double s_loss = block128_sum<double>(act ? (double)tl : 0.0, shd);
+  const double s_ratio = block128_sum<double>(act ? (double)ratio : 0.0, shd);
+  const double s_ent = block128_sum<double>(act ? (double)ent : 0.0, shd);
+  const double m_alr = block128_max(alr, shd);
+  const long long c_lo = block128_sum<long long>(clip_lo_hit, shl);
+  const long long c_hi = block128_sum<long long>(clip_hi_hit, shl);
+  if (threadIdx.x == 0) {
+    tile_flag[blockIdx.x] = any ? 1 : 0;
+    r[0] = s_loss;
+    r[1] = s_ratio;
+    r[2] = s_ent;
+    r[3] = m_alr;
+    r[4] = static_cast<double>(c_lo);
+    r[5] = static_cast<double>(c_hi);
+  }
+}
+
+struct StatsDev {
+  double denom, loss, sum_ratio, sum_entropy, max_abs_log_ratio;
+  long long n_active, n_clip_low, n_clip_high;
+};
+
+// fixed-order reduction of the per-tile partials, the loss scalar, the stats
+// and the list of tiles whose rows have a nonzero gradient coefficient
+__global__ void __launch_bounds__(1024) finalize_kernel(double denom, int32_t* __restrict__ counts,
+                                                        const int32_t* __restrict__ tile_flag,
+                                                        int32_t* __restrict__ tile_list,
+                                                        const double* __restrict__ red, float* __restrict__ loss_out,
+                                                        StatsDev* __restrict__ stats, unsigned* err) {
+  __shared__ double sh[6][32];
+  const int n = counts[0];
+  const int n_tiles = (n + kTileM - 1) / kTileM;
+  double a[6] = {0, 0, 0, 0, 0, 0};
+  for (int b = threadIdx.x; b < n_tiles; b += blockDim.x) {
+    const double* r = red + (int64_t)b * kRedSlots;
+    a[0] += r[0];
+    a[1] += r[1];
+    a[2] += r[2];
+    a[3] = fmax(a[3], r[3]);
+    a[4] += r[4];
+    a[5] += r[5];
+  }
+  // fixed shuffle tree inside each warp, then warp 0 over the 32 warp results
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+    for (int q = 0; q < 6; ++q) {
+      const double y = __shfl_xor_sync(0xffffffffu, a[q], o);
+      a[q] = (q == 3) ? fmax(a[q], y) : a[q] + y;
+    }
+  }
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (lane == 0)
+    for (int q = 0; q < 6; ++q) sh[q][w] = a[q];
+  __syncthreads();
+  if (w == 0) {
+    for (int q = 0; q < 6; ++q) a[q] = sh[q][lane];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+#pragma unroll
+      for (int q = 0; q < 6; ++q) {
+        const double y = __shfl_xor_sync(0xffffffffu, a[q], o);
+        a[q] = (q == 3) ? fmax(a[q], y) : a[q] + y;
+      }
+    }
+    if (lane == 0)
+      for (int q = 0; q < 6; ++q) sh[q][0] = a[q];
+  }
+  __syncthreads();
+  const double D = denom > 0.0 ? denom : static_cast<double>(n);
+  if (threadIdx.x == 0) {
+    if (!(D > 0.0)) atomicOr(err, kDevErrZeroDenom);
+    const double loss = D > 0.0 ? sh[0][0] / D : 0.0;
+    if (loss_out) *loss_out = static_cast<float>(loss);
+    if (stats) {
+      stats->denom = D;
+      stats->loss = loss;
+      stats->sum_ratio = sh[1][0];
+      stats->sum_entropy = sh[2][0];
+      stats->max_abs_log_ratio = sh[3][0];
+      stats->n_active = n;
+      stats->n_clip_low = static_cast<long long>(sh[4][0]);
+      stats->n_clip_high = static_cast<long long>(sh[5][0]);
+    }
+  }
+  // compact the active tile list (order preserving)
+  const int per = (n_tiles + blockDim.x - 1) / blockDim.x;
+  const int b0 = threadIdx.x * per, b1 = min(n_tiles, b0 + per);
+  int c = 0;
+  for (int b = b0; b < b1; ++b) c += tile_flag[b] ? 1 : 0;
+  int total;
+  int k = block_exclusive_scan(c, &total);
+  for (int b = b0; b < b1; ++b)
+    if (tile_flag[b]) tile_list[k++] = b;
+  if (threadIdx.x == 0) counts[1] = total;
+}
+
+// dhidden_out[t] = bf16(dh32[pos[t]]) for active rows, 0 for masked rows
+__global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __restrict__ pos, int T, int H,
+                               uint16_t* __restrict__ out) {
+  const int vpr = H / 8;
+  const int64_t total = (int64_t)T * vpr;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int t = (int)(i / vpr), v = (int)(i - (int64_t)t * vpr);
+    const int k = pos[t];
+    uint4 o = make_uint4(0, 0, 0, 0);
+    if (k >= 0) {
+      const float4* src = reinterpret_cast<const float4*>(dh32 + (int64_t)k * H) + 2 * v;
+      const float4 a = src[0], c = src[1];
+      o.x = pack_bf16x2(a.x, a.y);
+      o.y = pack_bf16x2(a.z, a.w);
+      o.z = pack_bf16x2(c.x, c.y);
+      o.w = pack_bf16x2(c.z, c.w);
+    }
+    reinterpret_cast<uint4*>(out + (int64_t)t * H)[v] = o;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
+                                    unsigned* err, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int threads = 256;
+  const int blocks = (int)(((int64_t)n * 32 + threads - 1) / threads);
+  group_adv_kernel<<<blocks, threads, 0, s>>>(rewards, gids, n, eps, out, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_broadcast(const float* adv, const int32_t* rot, int n_resp, int T, float* out, cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  const int blocks = min((T + 255) / 256, 4096);
+  broadcast_kernel<<<blocks, 256, 0, s>>>(adv, rot, n_resp, T, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_mask_count(const uint8_t* mask, int64_t T, int64_t* out, cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(out, 0, sizeof(int64_t), s);
+  if (e != cudaSuccess || T <= 0) return e;
+  const int64_t nb = (T / 16 + 255) / 256 + 1;
+  const int blocks = (int)(nb < 1024 ? nb : 1024);
+  mask_count_kernel<<<blocks, 256, 0, s>>>(mask, T, reinterpret_cast<unsigned long long*>(out));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compact(const uint8_t* mask, int T, const Workspace& ws, cudaStream_t s) {
+  compact_kernel<<<1, 1024, 0, s>>>(mask, T, ws.row_map, ws.pos_of_row, ws.counts);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const uint16_t* hidden, const int32_t* tokens, const float* b, const float* adv, int T,
+                          int Tcap, int H, const Workspace& ws, int n_sm, cudaStream_t s) {
+  (void)T;
+  gather_kernel<<<n_sm * 8, 256, 0, s>>>(hidden, tokens, b, adv, Tcap, H, ws.row_map, ws.counts, ws.h_p, ws.tok_p,
+                                         b ? ws.b_p : nullptr, adv ? ws.adv_p : nullptr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge(bool loss_mode, int Tcap, int V, int n_split, double denom, float clip_lo, float clip_hi,
+                         const Workspace& ws, float* logp_out, float* ent_out, float* tokloss_out, unsigned* err,
+                         cudaStream_t s) {
+  const int blocks = Tcap / kTileM;
+  merge_kernel<<<blocks, kTileM, 0, s>>>(loss_mode ? 1 : 0, Tcap, V, n_split, denom, clip_lo, clip_hi, ws.counts,
+                                          ws.row_map, ws.tok_p, ws.b_p, ws.adv_p, ws.part, ws.zx, ws.lse, ws.coef,
+                                          ws.tile_flag, ws.red, logp_out, ent_out, tokloss_out, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* loss_out, void* stats_out,
+                            unsigned* err, cudaStream_t s) {
+  (void)Tcap;
+  finalize_kernel<<<1, 1024, 0, s>>>(denom, ws.counts, ws.tile_flag, ws.tile_list, ws.red, loss_out,
+                                     reinterpret_cast<StatsDev*>(stats_out), err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  cast_dh_kernel<<<n_sm * 8, 256, 0, s>>>(ws.dh32, ws.pos_of_row, T, H, dh_out);
+  return cudaGetLastError();
+}
+
+}  // namespace molt

@@ -1,0 +1,75 @@
+"""CPU-side checks of the C ABI: the library builds for sm_103a, loads, exports
+every function include/molt.h declares, and rejects bad arguments on the host
+before touching a device."""
+import ctypes
+
+import pytest
+
+import paper_2607_21653_gb300 as molt
+
+
+@pytest.fixture(scope="module")
+def lib():
+    molt.build()
+    return molt.load()
+
+
+def test_exports_every_header_function(lib):
+    names = molt.header_functions()
+    assert "molt_policy_loss_fwd_bwd" in names and "molt_group_advantages" in names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings(lib):
+    for code in molt.STATUS:
+        s = lib.molt_status_string(code).decode()
+        assert s and s != "unknown status"
+    assert lib.molt_version() >= 1
+
+
+FAKE = 0x1000  # never dereferenced: every call below fails validation first
+
+
+def test_rejects_unsupported_hidden(lib):
+    st = lib.molt_token_logprobs_fwd(FAKE, FAKE, FAKE, None, 16, 100, 32, FAKE, None, None, 0, None)
+    assert molt.STATUS[st] == "MOLT_ERR_UNSUPPORTED_SHAPE"
+    assert "multiple of 64" in lib.molt_last_error().decode()
+
+
+def test_rejects_null_and_misaligned(lib):
+    st = lib.molt_token_logprobs_fwd(None, FAKE, FAKE, None, 16, 64, 32, FAKE, None, None, 0, None)
+    assert molt.STATUS[st] == "MOLT_ERR_INVALID_ARG"
+    st = lib.molt_token_logprobs_fwd(FAKE + 2, FAKE, FAKE, None, 16, 64, 32, FAKE, None, None, 0, None)
+    assert molt.STATUS[st] == "MOLT_ERR_INVALID_ARG"
+    st = lib.molt_mask_count(FAKE + 1, 64, FAKE, None)
+    assert molt.STATUS[st] == "MOLT_ERR_INVALID_ARG"
+
+
+def test_rejects_bad_clip_and_sizes(lib):
+    args = [FAKE] * 6 + [16, 64, 32, 1.5, 0.2, 0.0] + [FAKE, FAKE, FAKE, 0, None, None, None, None, None, 0, None]
+    st = lib.molt_policy_loss_fwd_bwd(*args)
+    assert molt.STATUS[st] == "MOLT_ERR_INVALID_ARG"
+    args[9] = 0.2
+    args[11] = float("nan")
+    assert molt.STATUS[lib.molt_policy_loss_fwd_bwd(*args)] == "MOLT_ERR_INVALID_ARG"
+    args[11] = 0.0
+    args[6] = -1
+    assert molt.STATUS[lib.molt_policy_loss_fwd_bwd(*args)] == "MOLT_ERR_INVALID_ARG"
+    assert molt.STATUS[lib.molt_group_advantages(FAKE, FAKE, -3, 1e-6, FAKE, None)] == "MOLT_ERR_INVALID_ARG"
+    assert molt.STATUS[lib.molt_group_advantages(FAKE, FAKE, 4, -1.0, FAKE, None)] == "MOLT_ERR_INVALID_ARG"
+
+
+def test_empty_inputs_are_noops(lib):
+    assert lib.molt_group_advantages(None, None, 0, 1e-6, None, None) == 0
+    assert lib.molt_broadcast_advantages(None, None, 0, 0, None, None) == 0
+    assert lib.molt_token_logprobs_fwd(FAKE, FAKE, FAKE, None, 0, 64, 32, FAKE, None, None, 0, None) == 0
+
+
+def test_workspace_sizes_grow_with_problem(lib):
+    a = molt.token_logprobs_workspace_bytes(1000, 256, 4096)
+    b = molt.policy_loss_workspace_bytes(1000, 256, 4096)
+    assert 0 < a < b
+    assert molt.policy_loss_workspace_bytes(1000, 100, 4096) == 0   # unsupported H
+    # dhidden fp32 accumulator + packed bf16 copy of the hidden rows dominate
+    assert b >= 1024 * 256 * 6
