@@ -155,6 +155,21 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
                                      float* token_loss_out, molt_stats* stats_out, void* workspace,
                                      size_t workspace_bytes, cudaStream_t stream);
 
+/*
+ * Per-kernel timing hook for benchmarks.  While set, every LM-head call made
+ * from the calling thread records starts[k] / stops[k] (caller-created CUDA
+ * events) on its stream around kernel group k:
+ *   k = 0  active-row compaction and packed gather
+ *   k = 1  LM-head forward kernel (online log-softmax)
+ *   k = 2  split merge, surrogate loss and the fixed-order reductions
+ *   k = 3  LM-head backward kernel (dhidden / dW products)
+ *   k = 4  dhidden cast
+ * Slots beyond n are ignored.  n = 0 (or NULL arrays) turns the hook off.
+ * The arrays are read at each call, not copied: keep them alive while set.
+ */
+#define MOLT_TIMING_SLOTS 5
+void molt_set_timing_events(cudaEvent_t* starts, cudaEvent_t* stops, int n);
+
 #ifdef __cplusplus
 }
 #endif

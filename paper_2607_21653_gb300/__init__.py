@@ -117,6 +117,7 @@ def load():
         "molt_policy_loss_workspace_bytes": (SZ, [I64, I64, I64]),
         "molt_policy_loss_fwd_bwd": (I32, [P, P, P, P, P, P, I64, I64, I64, F, F, D, P, P, P, I32, P, P, P, P,
                                             P, SZ, P]),
+        "molt_set_timing_events": (None, [P, P, I32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -124,6 +125,42 @@ def load():
         fn.argtypes = args
     _lib = L
     return L
+
+
+TIMING_SLOTS = ("gather", "forward", "merge", "backward", "cast")
+
+
+class KernelTimer:
+    """Records CUDA events around the library's kernel groups (C-ABI timing hook)
+    for a series of steps; `elapsed_ms()` sums each group's time over the steps."""
+
+    def __init__(self, steps: int):
+        torch = _torch()
+        n = len(TIMING_SLOTS)
+        self.ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+                   for _ in range(steps)]
+        self._arrays = []
+
+    def arm(self, step: int):
+        n = len(TIMING_SLOTS)
+        starts = (ctypes.c_void_p * n)(*[e[0].cuda_event for e in self.ev[step]])
+        stops = (ctypes.c_void_p * n)(*[e[1].cuda_event for e in self.ev[step]])
+        self._arrays.append((starts, stops))
+        load().molt_set_timing_events(starts, stops, n)
+
+    @staticmethod
+    def disarm():
+        load().molt_set_timing_events(None, None, 0)
+
+    def elapsed_ms(self) -> dict:
+        out = {k: 0.0 for k in TIMING_SLOTS}
+        for step in self.ev:
+            for k, (a, b) in zip(TIMING_SLOTS, step):
+                try:
+                    out[k] += a.elapsed_time(b)
+                except RuntimeError:
+                    pass
+        return out
 
 
 def header_functions() -> list[str]:

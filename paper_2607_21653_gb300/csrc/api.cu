@@ -22,6 +22,18 @@ namespace {
 
 thread_local std::string t_last_error;
 
+// benchmark timing hook (molt_set_timing_events)
+thread_local cudaEvent_t* t_ev_start = nullptr;
+thread_local cudaEvent_t* t_ev_stop = nullptr;
+thread_local int t_ev_n = 0;
+
+inline void ev_start(int k, cudaStream_t s) {
+  if (k < t_ev_n && t_ev_start && t_ev_start[k]) cudaEventRecord(t_ev_start[k], s);
+}
+inline void ev_stop(int k, cudaStream_t s) {
+  if (k < t_ev_n && t_ev_stop && t_ev_stop[k]) cudaEventRecord(t_ev_stop[k], s);
+}
+
 molt_status fail(molt_status s, const std::string& msg) {
   t_last_error = msg;
   return s;
@@ -221,10 +233,12 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
                         const float* b, const float* adv, int64_t T, int64_t H, int64_t V, int S,
                         const Workspace& w, const CUtensorMap& tm_h, const CUtensorMap& tm_w, cudaStream_t s) {
   const int64_t Tcap = round_tiles(T);
+  ev_start(0, s);
   MOLT_CUDA(launch_compact(mask, static_cast<int>(T), w, s), "compact");
   MOLT_CUDA(launch_gather(hidden, tokens, b, adv, static_cast<int>(T), static_cast<int>(Tcap), static_cast<int>(H),
                           w, di->n_sm, s),
             "gather");
+  ev_stop(0, s);
   FwdArgs fa{};
   fa.tok_p = w.tok_p;
   fa.counts = w.counts;
@@ -236,7 +250,9 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
   fa.part = w.part;
   fa.zx = w.zx;
   fa.err = di->status;
+  ev_start(1, s);
   MOLT_CUDA(launch_lmhead_fwd(tm_h, tm_w, fa, di->n_sm, s), "lmhead forward");
+  ev_stop(1, s);
   return MOLT_OK;
 }
 
@@ -266,6 +282,12 @@ const char* molt_status_string(molt_status s) {
 const char* molt_last_error(void) { return t_last_error.c_str(); }
 
 int molt_version(void) { return 1; }
+
+void molt_set_timing_events(cudaEvent_t* starts, cudaEvent_t* stops, int n) {
+  t_ev_start = starts;
+  t_ev_stop = stops;
+  t_ev_n = (starts && stops && n > 0) ? n : 0;
+}
 
 molt_status molt_device_status(cudaStream_t stream, uint32_t* flags) {
   if (!flags) return fail(MOLT_ERR_INVALID_ARG, "flags is NULL");
@@ -359,9 +381,11 @@ molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, c
   MOLT_TRY(run_forward(di, hidden, tokens, mask, nullptr, nullptr, T, H, V, S, w, tm_h, tm_w, stream));
   MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
   if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
+  ev_start(2, stream);
   MOLT_CUDA(launch_merge(false, static_cast<int>(Tcap), static_cast<int>(V), S, 0.0, 0.f, 0.f, w, logp_out,
                          entropy_out, nullptr, di->status, stream),
             "merge");
+  ev_stop(2, stream);
   return MOLT_OK;
 }
 
@@ -407,10 +431,12 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
   if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
   if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
   if (token_loss_out) MOLT_CUDA(cudaMemsetAsync(token_loss_out, 0, T * sizeof(float), stream), "memset token loss");
+  ev_start(2, stream);
   MOLT_CUDA(launch_merge(true, static_cast<int>(Tcap), static_cast<int>(V), S, denom, clip_lo, clip_hi, w, logp_out,
                          entropy_out, token_loss_out, di->status, stream),
             "merge");
   MOLT_CUDA(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, di->status, stream), "finalize");
+  ev_stop(2, stream);
   MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
   if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
   BwdArgs ba{};
@@ -424,8 +450,12 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
   ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
   ba.tile_group = 16;
   ba.err = di->status;
+  ev_start(3, stream);
   MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  ev_stop(3, stream);
+  ev_start(4, stream);
   MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
+  ev_stop(4, stream);
   return MOLT_OK;
 }
 
