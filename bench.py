@@ -259,6 +259,7 @@ def run_ours(args):
     clk = clocks.stop()
     ms = t0.elapsed_time(t1)
     per = timer.elapsed_ms()
+    timer.close()
     assert molt.device_status() == 0
     loss_val = float(out["loss"].item())
     if world > 1:

@@ -130,21 +130,39 @@ def load():
 TIMING_SLOTS = ("gather", "forward", "merge", "backward", "cast")
 
 
+def _cudart():
+    """The CUDA runtime already loaded in this process (libmolt links it)."""
+    load()
+    rt = ctypes.CDLL("libcudart.so.13")
+    rt.cudaEventCreate.argtypes = [ctypes.POINTER(ctypes.c_void_p)]
+    rt.cudaEventElapsedTime.argtypes = [ctypes.POINTER(ctypes.c_float), ctypes.c_void_p, ctypes.c_void_p]
+    rt.cudaEventDestroy.argtypes = [ctypes.c_void_p]
+    return rt
+
+
 class KernelTimer:
     """Records CUDA events around the library's kernel groups (C-ABI timing hook)
-    for a series of steps; `elapsed_ms()` sums each group's time over the steps."""
+    for a series of steps; `elapsed_ms()` sums each group's time over the steps.
+    The events are raw cudaEvent_t handles created through the CUDA runtime."""
 
     def __init__(self, steps: int):
-        torch = _torch()
+        self.rt = _cudart()
         n = len(TIMING_SLOTS)
-        self.ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
-                   for _ in range(steps)]
+        self.ev = []
+        for _ in range(steps):
+            row = []
+            for _ in range(n):
+                a, b = ctypes.c_void_p(), ctypes.c_void_p()
+                if self.rt.cudaEventCreate(ctypes.byref(a)) or self.rt.cudaEventCreate(ctypes.byref(b)):
+                    raise RuntimeError("cudaEventCreate failed")
+                row.append((a, b))
+            self.ev.append(row)
         self._arrays = []
 
     def arm(self, step: int):
         n = len(TIMING_SLOTS)
-        starts = (ctypes.c_void_p * n)(*[e[0].cuda_event for e in self.ev[step]])
-        stops = (ctypes.c_void_p * n)(*[e[1].cuda_event for e in self.ev[step]])
+        starts = (ctypes.c_void_p * n)(*[e[0].value for e in self.ev[step]])
+        stops = (ctypes.c_void_p * n)(*[e[1].value for e in self.ev[step]])
         self._arrays.append((starts, stops))
         load().molt_set_timing_events(starts, stops, n)
 
@@ -153,14 +171,21 @@ class KernelTimer:
         load().molt_set_timing_events(None, None, 0)
 
     def elapsed_ms(self) -> dict:
+        """Call after the stream has been synchronised."""
         out = {k: 0.0 for k in TIMING_SLOTS}
-        for step in self.ev:
-            for k, (a, b) in zip(TIMING_SLOTS, step):
-                try:
-                    out[k] += a.elapsed_time(b)
-                except RuntimeError:
-                    pass
+        ms = ctypes.c_float()
+        for row in self.ev:
+            for k, (a, b) in zip(TIMING_SLOTS, row):
+                if self.rt.cudaEventElapsedTime(ctypes.byref(ms), a, b) == 0:
+                    out[k] += ms.value
         return out
+
+    def close(self):
+        for row in self.ev:
+            for a, b in row:
+                self.rt.cudaEventDestroy(a)
+                self.rt.cudaEventDestroy(b)
+        self.ev = []
 
 
 def header_functions() -> list[str]:
