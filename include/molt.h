@@ -156,6 +156,36 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
                                      size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * Allocation-free variant of molt_token_logprobs_fwd (the paper has no
+ * counterpart; it exists for callers, not for the method).
+ *
+ * Some callers cannot let a library allocate device memory: a training or
+ * serving runtime that reserves the GPU's memory up front and hands it out only
+ * through its own pool, or a process whose memory budget leaves nothing outside
+ * that pool.  This call allocates nothing (no cudaMalloc, cudaMallocAsync or
+ * cudaFree).  Its scratch is one fixed device array of about 4 MB, sized for
+ * MOLT_NOALLOC_MAX_TOKENS tokens, that every GPU which loads the library keeps
+ * until the process exits.  The caller still owns and passes all inputs and
+ * outputs, with the same meaning as in molt_token_logprobs_fwd.
+ *   - T > MOLT_NOALLOC_MAX_TOKENS returns MOLT_ERR_UNSUPPORTED_SHAPE and
+ *     launches nothing; split larger batches into several calls.
+ *   - All calls on a device share the one scratch array and each call leaves
+ *     its contents behind (the call clears what it needs before use).  Calls
+ *     whose kernels may overlap on the GPU (different streams, or different
+ *     host threads, without ordering between them) race on that array: order
+ *     them, e.g. by issuing them on one stream.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); later calls reuse it.
+ *     Make the first call on a device before any stream capture on it.
+ * Masked rows are computed and then written as 0 (there is no compaction),
+ * so prefer molt_token_logprobs_fwd when allocation is allowed.
+ */
+#define MOLT_NOALLOC_MAX_TOKENS 32768
+molt_status molt_token_logprobs_fwd_noalloc(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                                            const uint8_t* mask, int64_t T, int64_t H, int64_t V,
+                                            float* logp_out, float* entropy_out, cudaStream_t stream);
+
+/*
  * Per-kernel timing hook for benchmarks.  While set, every LM-head call made
  * from the calling thread records starts[k] / stops[k] (caller-created CUDA
  * events) on its stream around kernel group k:

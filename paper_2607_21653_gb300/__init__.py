@@ -28,7 +28,7 @@ _CSRC = os.path.join(_PKG, "csrc")
 _INCLUDE = os.path.join(_ROOT, "include")
 _BUILD = os.path.join(_ROOT, "_build")
 _LIB = os.path.join(_PKG, "libmolt.so")
-_SOURCES = ["rows.cu", "lmhead_fwd.cu", "lmhead_bwd.cu", "api.cu"]
+_SOURCES = ["rows.cu", "lmhead_fwd.cu", "lmhead_bwd.cu", "api.cu", "noalloc.cu"]
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 STATUS = {
@@ -118,6 +118,7 @@ def load():
         "molt_policy_loss_fwd_bwd": (I32, [P, P, P, P, P, P, I64, I64, I64, F, F, D, P, P, P, I32, P, P, P, P,
                                             P, SZ, P]),
         "molt_set_timing_events": (None, [P, P, I32]),
+        "molt_token_logprobs_fwd_noalloc": (I32, [P, P, P, P, I64, I64, I64, P, P, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -307,6 +308,24 @@ def token_logprobs(hidden, weight, tokens, mask=None, want_entropy=True, stream=
                                           _ptr(tokens, torch.int32, "tokens"), _ptr(mask, torch.uint8, "mask"),
                                           T, H, V, _ptr(logp), _ptr(ent), ws.data_ptr(), ws.numel(),
                                           _stream(stream)))
+    return logp, ent
+
+
+NOALLOC_MAX_TOKENS = 32768
+
+
+def token_logprobs_noalloc(hidden, weight, tokens, mask=None, want_entropy=True, stream=None):
+    """Like token_logprobs, through molt_token_logprobs_fwd_noalloc: the library
+    allocates nothing (its scratch is a fixed device array); T <= 32768."""
+    torch = _torch()
+    T, H = hidden.shape
+    V = weight.shape[0]
+    logp = torch.empty(T, dtype=torch.float32, device=hidden.device)
+    ent = torch.empty(T, dtype=torch.float32, device=hidden.device) if want_entropy else None
+    _check(load().molt_token_logprobs_fwd_noalloc(_bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"),
+                                                  _ptr(tokens, torch.int32, "tokens"),
+                                                  _ptr(mask, torch.uint8, "mask"), T, H, V, _ptr(logp), _ptr(ent),
+                                                  _stream(stream)))
     return logp, ent
 
 

@@ -257,6 +257,25 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
 }
 
 }  // namespace
+
+void set_last_error(const std::string& msg) { t_last_error = msg; }
+
+unsigned* device_status_word(molt_status* st) {
+  const DeviceInfo* di = device_info(st);
+  return di ? di->status : nullptr;
+}
+
+int device_sm_count() {
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  return di ? di->n_sm : 1;
+}
+
+molt_status encode_tmap_2d(CUtensorMap* m, CUtensorMapDataType dt, int elem_bytes, const void* base, uint64_t rows,
+                           uint64_t cols, uint32_t box_cols, uint32_t box_rows) {
+  return make_tmap(m, dt, elem_bytes, base, rows, cols, box_cols, box_rows);
+}
+
 }  // namespace molt
 
 using namespace molt;

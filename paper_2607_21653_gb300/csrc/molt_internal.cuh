@@ -4,6 +4,9 @@
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <string>
+
+#include "../../include/molt.h"
 
 namespace molt {
 
@@ -55,6 +58,13 @@ struct BwdArgs {
   int tile_group;            // token tiles per raster group
   unsigned* err;
 };
+
+// api.cu: shared host helpers
+void set_last_error(const std::string& msg);
+unsigned* device_status_word(molt_status* st);   // current device's status word
+int device_sm_count();                           // current device's SM count
+molt_status encode_tmap_2d(CUtensorMap* m, CUtensorMapDataType dt, int elem_bytes, const void* base, uint64_t rows,
+                           uint64_t cols, uint32_t box_cols, uint32_t box_rows);
 
 // rows.cu
 cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
