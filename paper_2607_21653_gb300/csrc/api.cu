@@ -439,10 +439,11 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
   Scratch sc;
   MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
   const Workspace w = carve(sc.ptr, L);
+  const bool pair_bwd = (H % 256) == 0;
   CUtensorMap tm_h, tm_w, tm_wz, tm_wn, tm_dh, tm_dw;
   MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
   MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
-  MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kBwdBV));
+  MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, pair_bwd ? 128 : kBwdBV));
   MOLT_TRY(make_tmap(&tm_wn, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, 64));
   MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
   MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
@@ -467,10 +468,13 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
   ba.V = static_cast<int>(V);
   ba.H = static_cast<int>(H);
   ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
-  ba.tile_group = 16;
+  ba.tile_group = pair_bwd ? 8 : 16;
   ba.err = di->status;
   ev_start(3, stream);
-  MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  if (pair_bwd)
+    MOLT_CUDA(launch_lmhead_bwd_pair(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  else
+    MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
   ev_stop(3, stream);
   ev_start(4, stream);
   MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");

@@ -136,10 +136,18 @@ def _check_loss(out, ref, m):
 
 
 LOSS_SHAPES = [
+    # single-CTA backward (H not a multiple of 256)
     (300, 128, 1000, 0.2),
     (513, 192, 4133, 0.3),
     (256, 320, 2304, 0.0),
     (1, 64, 7, 0.0),
+    # CTA-pair backward (H a multiple of 256): odd and even tile counts, a pair
+    # whose second CTA has no tile, several H chunks, ragged vocab tails
+    (300, 256, 1000, 0.2),
+    (513, 512, 4133, 0.3),
+    (1, 256, 7, 0.0),
+    (640, 768, 2304, 0.0),
+    (1000, 256, 5000, 0.6),
 ]
 
 
