@@ -20,12 +20,19 @@
 //           GW = all 256 tokens x 128 vocab of one half (MN-major A of dW).  The
 //           GW rows for the peer's vocab half are written into the peer's
 //           shared memory (distributed shared memory).
-//   job dH  per 256 columns of H: pair MMA M=256 tokens, N=256, K=256 vocab;
-//           B = W_j rows, MN-major, CTA r staging columns 128 r .. 128 r + 127.
-//   job dW  per 256 columns of H: pair MMA M=256 vocab (CTA r: half r),
-//           N=256, K=256 tokens; B = h rows of both tiles, MN-major.
+//   job dH  per 128 columns of H: pair MMA M=256 tokens, N=128, K=256 vocab;
+//           B = W_j rows, MN-major, CTA r staging columns 64 r .. 64 r + 63.
+//   job dW  per 128 columns of H: pair MMA M=256 vocab (CTA r: half r),
+//           N=128, K=256 tokens; B = h rows of both tiles, MN-major.
 // Partial products drain through swizzled 32 x 32 fp32 boxes with TMA
 // reduce-add into the fp32 dhidden accumulator and dW.
+//
+// Schedule.  Each SM can push only ~25 B/clock of reduce-adds to L2, and a
+// unit's drains (4 B x H x 256 per CTA) take longer than its products, so the
+// drain path must never idle.  TMEM holds one 256-column Z buffer and a ring of
+// two 128-column job accumulators; the MMA issuer interleaves the K-blocks of
+// the NEXT unit's Z between the current unit's dH/dW jobs (H/64 of each, one
+// after the other), so the next logits accumulate while the epilogue drains.
 //
 // Roles per CTA (192 threads): warp 0 TMA producer (both CTAs load their
 // halves; bytes complete on the even CTA's barrier), warp 1 MMA issuer (even
@@ -52,8 +59,10 @@ constexpr int kBoxesPerWarp = 2;
 constexpr int kThreads = 192;
 constexpr int kSmemBytes = 1024 + kOffBox + 4 * kBoxesPerWarp * kBoxBytes;
 constexpr uint32_t kIdescZ = idesc_bf16_f32(256, 256, false, false);
-constexpr uint32_t kIdescH = idesc_bf16_f32(256, 256, false, true);
-constexpr uint32_t kIdescW = idesc_bf16_f32(256, 256, true, true);
+constexpr uint32_t kIdescH = idesc_bf16_f32(256, 128, false, true);
+constexpr uint32_t kIdescW = idesc_bf16_f32(256, 128, true, true);
+constexpr uint32_t kZCol = 0;      // TMEM columns [0, 256): Z buffer
+constexpr uint32_t kAccCol = 256;  // [256, 384), [384, 512): job accumulators
 constexpr uint32_t kStageTx = 2u * kStageBytes;   // bytes both CTAs load per stage
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -90,9 +99,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kStages];    // even CTA: both CTAs' bytes land here
   __shared__ __align__(8) uint64_t empty_bar[kStages];   // both CTAs, committed by the even CTA
-  __shared__ __align__(8) uint64_t accf_bar[2];          // both CTAs, committed by the even CTA
+  __shared__ __align__(8) uint64_t accf_bar[2];          // both CTAs: job accumulator full
   __shared__ __align__(8) uint64_t acce_bar[2];          // even CTA: 256 epilogue arrivals
-  __shared__ __align__(8) uint64_t gready_bar;           // even CTA: 256 epilogue arrivals
+  __shared__ __align__(8) uint64_t zfull_bar;            // both CTAs: Z buffer complete
+  __shared__ __align__(8) uint64_t gready_bar;           // even CTA: g written, Z buffer read (256)
   __shared__ __align__(8) uint64_t done_bar;
   __shared__ uint32_t tmem_base_sh;
   __shared__ int abort_sh;
@@ -116,6 +126,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&accf_bar[b]), 1);
       mbar_init(smem_u32(&acce_bar[b]), 256);
     }
+    mbar_init(smem_u32(&zfull_bar), 1);
     mbar_init(smem_u32(&gready_bar), 256);
     mbar_init(smem_u32(&done_bar), 1);
     abort_sh = 0;
@@ -136,8 +147,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
   const int n_vc = a.n_vchunks;
   const int n_units = n_tp * n_vc;
   const int H = a.H, V = a.V;
-  const int kblocks = H / kBK;
-  const int nC = H / 256;
+  const int nZ = H / kBK;        // Z K-blocks per unit
+  const int nJ = H / kBK;        // jobs per unit: H/128 dH jobs, then H/128 dW jobs
+  const int nJH = H / 128;
   const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
 
   if (warp == 0) {
@@ -159,34 +171,43 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         ++it;
         return true;
       };
-      for (int u = pair; u < n_units && ok; u += n_pairs) {
+      auto rows_of = [&](int u, int& ta, int& tb, int& v0) {
         const PairUnit un = pair_unit_of(u, n_tp, n_vc, a.tile_group);
-        const int ta = a.tile_list[2 * un.tp];
-        const int tb = (2 * un.tp + 1 < n_tiles) ? a.tile_list[2 * un.tp + 1] : ta;
-        const int own_row0 = (rank ? tb : ta) * kTileM;
-        const int v0 = un.vc * 256;
+        ta = a.tile_list[2 * un.tp];
+        tb = (2 * un.tp + 1 < n_tiles) ? a.tile_list[2 * un.tp + 1] : ta;
+        v0 = un.vc * 256;
+      };
+      auto load_z = [&](int kb, int own_row0, int v0) -> bool {
         uint32_t sa, fb;
-        for (int kb = 0; kb < kblocks && ok; ++kb) {
+        if (!next_stage(sa, fb)) return false;
+        tma_load_2d_pair(sa, &tm_h, fb, kb * kBK, own_row0);
+        tma_load_2d_pair(sa + kSub, &tm_wz, fb, kb * kBK, v0 + static_cast<int>(rank) * 128);
+        return true;
+      };
+      int u = pair;
+      if (u < n_units) {
+        int ta, tb, v0;
+        rows_of(u, ta, tb, v0);
+        for (int kb = 0; kb < nZ && ok; ++kb) ok = load_z(kb, (rank ? tb : ta) * kTileM, v0);
+      }
+      for (; u < n_units && ok; u += n_pairs) {
+        int ta, tb, v0;
+        rows_of(u, ta, tb, v0);
+        const int un_next = u + n_pairs;
+        int nta = 0, ntb = 0, nv0 = 0;
+        if (un_next < n_units) rows_of(un_next, nta, ntb, nv0);
+        for (int i = 0; i < nJ && ok; ++i) {
+          uint32_t sa, fb;
           if (!(ok = next_stage(sa, fb))) break;
-          tma_load_2d_pair(sa, &tm_h, fb, kb * kBK, own_row0);
-          tma_load_2d_pair(sa + kSub, &tm_wz, fb, kb * kBK, v0 + static_cast<int>(rank) * 128);
-        }
-        for (int nc = 0; nc < nC && ok; ++nc) {
-          for (int half = 0; half < 2 && ok; ++half) {
-            if (!(ok = next_stage(sa, fb))) break;
-            for (int vb = 0; vb < 2; ++vb)
-              for (int q = 0; q < 2; ++q)
-                tma_load_2d_pair(sa + vb * 16384 + q * 8192, &tm_wn, fb,
-                                 nc * 256 + static_cast<int>(rank) * 128 + q * 64, v0 + half * 128 + vb * 64);
+          if (i < nJH) {   // dH job: W rows v0 .. v0+255, this CTA's 64 of 128 columns
+            const int x = i * 128 + static_cast<int>(rank) * 64;
+            for (int vb = 0; vb < 4; ++vb) tma_load_2d_pair(sa + vb * 8192, &tm_wn, fb, x, v0 + vb * 64);
+          } else {         // dW job: h rows of both tiles, this CTA's 64 of 128 columns
+            const int x = (i - nJH) * 128 + static_cast<int>(rank) * 64;
+            tma_load_2d_pair(sa, &tm_h, fb, x, ta * kTileM);
+            tma_load_2d_pair(sa + 16384, &tm_h, fb, x, tb * kTileM);
           }
-        }
-        for (int nc = 0; nc < nC && ok; ++nc) {
-          for (int tt = 0; tt < 2 && ok; ++tt) {
-            if (!(ok = next_stage(sa, fb))) break;
-            for (int q = 0; q < 2; ++q)
-              tma_load_2d_pair(sa + q * 16384, &tm_h, fb, nc * 256 + static_cast<int>(rank) * 128 + q * 64,
-                               (tt ? tb : ta) * kTileM);
-          }
+          if (un_next < n_units) ok = load_z(i, (rank ? ntb : nta) * kTileM, nv0);
         }
       }
       if (leader) {
@@ -212,67 +233,57 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         umma_commit_pair_mc(smem_u32(&empty_bar[it % kStages]), 3);
         ++it;
       };
-      auto acquire_acc = [&](uint32_t& d) -> bool {
-        const uint32_t buf = jj & 1u, aph = (jj >> 1) & 1u;
-        if (!mbar_wait_cluster(smem_u32(&acce_bar[buf]), aph ^ 1u, abort_flag, a.err)) return false;
-        tc_fence_after();
-        d = tmem_base + buf * 256;
+      // one Z K-block into the Z buffer
+      auto z_block = [&](int kb) -> bool {
+        uint32_t sa;
+        if (!wait_stage(sa)) return false;
+        const uint64_t ad = sdesc_sw128(sa, 16, 1024);
+        const uint64_t bd = sdesc_sw128(sa + kSub, 16, 1024);
+#pragma unroll
+        for (int k = 0; k < kBK / 16; ++k)
+          umma_bf16_pair(tmem_base + kZCol, ad + 2u * k, bd + 2u * k, kIdescZ, (kb | k) != 0 ? 1u : 0u);
+        release_stage();
+        if (kb == nZ - 1) umma_commit_pair_mc(smem_u32(&zfull_bar), 3);
         return true;
       };
-      auto publish_acc = [&]() {
-        umma_commit_pair_mc(smem_u32(&accf_bar[jj & 1u]), 3);
-        ++jj;
-      };
-      for (int u = pair; u < n_units && ok; u += n_pairs) {
-        uint32_t d, sa;
-        // job Z
-        if (!(ok = acquire_acc(d))) break;
-        for (int kb = 0; kb < kblocks && ok; ++kb) {
-          if (!(ok = wait_stage(sa))) break;
-          const uint64_t ad = sdesc_sw128(sa, 16, 1024);
-          const uint64_t bd = sdesc_sw128(sa + kSub, 16, 1024);
-#pragma unroll
-          for (int k = 0; k < kBK / 16; ++k)
-            umma_bf16_pair(d, ad + 2u * k, bd + 2u * k, kIdescZ, (kb | k) != 0 ? 1u : 0u);
-          release_stage();
-        }
-        if (!ok) break;
-        publish_acc();
-        // both CTAs' g tiles (local and remote parts) must be in place
+      int u = pair;
+      if (u < n_units)
+        for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb);
+      for (; u < n_units && ok; u += n_pairs) {
+        const bool has_next = u + n_pairs < n_units;
+        // g of this unit in shared memory, and the Z buffer free again
         if (!(ok = mbar_wait_cluster(smem_u32(&gready_bar), unit_it & 1u, abort_flag, a.err))) break;
         tc_fence_after();
-        // jobs dH: A = g (own tokens, K-major), B = W rows (MN-major)
-        for (int nc = 0; nc < nC && ok; ++nc) {
-          if (!(ok = acquire_acc(d))) break;
-          for (int half = 0; half < 2 && ok; ++half) {
-            if (!(ok = wait_stage(sa))) break;
+        for (int i = 0; i < nJ && ok; ++i) {
+          const uint32_t buf = jj & 1u, aph = (jj >> 1) & 1u;
+          if (!(ok = mbar_wait_cluster(smem_u32(&acce_bar[buf]), aph ^ 1u, abort_flag, a.err))) break;
+          tc_fence_after();
+          const uint32_t d = tmem_base + kAccCol + buf * 128;
+          uint32_t sa;
+          if (!(ok = wait_stage(sa))) break;
+          if (i < nJH) {
+            // dH: A = g (own tokens x 256 vocab, K-major), B = W rows (MN-major)
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
+            for (int k = 0; k < 16; ++k) {
               const int vb = k >> 2, kk = k & 3;
-              const uint64_t ad = sdesc_sw128(gh_base + (half * 2 + vb) * kSub, 16, 1024) + 2u * kk;
-              const uint64_t bd = sdesc_sw128(sa + vb * 16384 + kk * 2048, 8192, 1024);
-              umma_bf16_pair(d, ad, bd, kIdescH, (half | k) != 0 ? 1u : 0u);
+              const uint64_t ad = sdesc_sw128(gh_base + vb * kSub, 16, 1024) + 2u * kk;
+              const uint64_t bd = sdesc_sw128(sa + vb * 8192 + kk * 2048, 8192, 1024);
+              umma_bf16_pair(d, ad, bd, kIdescH, k != 0 ? 1u : 0u);
             }
-            release_stage();
-          }
-          if (!ok) break;
-          publish_acc();
-        }
-        // jobs dW: A = g^T (this CTA's vocab half x 256 tokens, MN-major), B = h rows (MN-major)
-        for (int nc = 0; nc < nC && ok; ++nc) {
-          if (!(ok = acquire_acc(d))) break;
-          for (int tt = 0; tt < 2 && ok; ++tt) {
-            if (!(ok = wait_stage(sa))) break;
+          } else {
+            // dW: A = g^T (this CTA's 128 vocab x 256 tokens, MN-major), B = h rows (MN-major)
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
+            for (int k = 0; k < 16; ++k) {
+              const int tt = k >> 3, kk = k & 7;
               const uint64_t ad = sdesc_sw128(gw_base + (tt * 8 + kk) * 2048, kGWBlock, 1024);
-              const uint64_t bd = sdesc_sw128(sa + kk * 2048, 16384, 1024);
-              umma_bf16_pair(d, ad, bd, kIdescW, (tt | kk) != 0 ? 1u : 0u);
+              const uint64_t bd = sdesc_sw128(sa + tt * 16384 + kk * 2048, 16384, 1024);
+              umma_bf16_pair(d, ad, bd, kIdescW, k != 0 ? 1u : 0u);
             }
-            release_stage();
           }
-          if (!ok) break;
-          publish_acc();
+          release_stage();
+          umma_commit_pair_mc(smem_u32(&accf_bar[buf]), 3);
+          ++jj;
+          if (has_next) ok = z_block(i);
         }
         ++unit_it;
       }
@@ -288,20 +299,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     const uint32_t acce_leader1 = mapa_shared(smem_u32(&acce_bar[1]), 0);
     const uint32_t gready_leader = mapa_shared(smem_u32(&gready_bar), 0);
     const uint32_t gw_peer = mapa_shared(gw_base, peer);
-    uint32_t jj = 0, nbox = 0;
+    uint32_t jj = 0, nbox = 0, unit_it = 0;
     bool ok = true;
-    auto acquire_full = [&](uint32_t& taddr) -> bool {
-      const uint32_t buf = jj & 1u, aph = (jj >> 1) & 1u;
-      if (!mbar_wait(smem_u32(&accf_bar[buf]), aph, abort_flag, a.err)) return false;
-      tc_fence_after();
-      taddr = tmem_base + lane_off + buf * 256;
-      return true;
-    };
-    auto release = [&]() {
-      tc_fence_before();
-      mbar_arrive_cluster((jj & 1u) ? acce_leader1 : acce_leader0);
-      ++jj;
-    };
     // one [32 x 32] fp32 slab of this warp's rows -> reduce-add into global
     auto drain_slab = [&](const CUtensorMap* map, uint32_t taddr, int x, int y, bool issue) {
       float v[32];
@@ -312,9 +311,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       write_box32(box, lane, v);
       fence_proxy_async_smem();
       __syncwarp();
-      if (lane == 0 && issue) {
-        tma_reduce_add_2d(map, box, x, y);
-      }
+      if (lane == 0 && issue) tma_reduce_add_2d(map, box, x, y);
       if (lane == 0) bulk_commit_group();
       ++nbox;
     };
@@ -331,13 +328,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const float lseL = (coef != 0.f) ? a.lse[row] * kLog2e : 0.f;
       const int lx = a.tok_p[row] - v0;
       const int R = static_cast<int>(rank) * 128 + r_in;   // row of this token in GW
-      uint32_t taddr;
-      // job Z -> g in GH (own tokens x 256 vocab) and GW (this / the peer CTA)
-      if (!(ok = acquire_full(taddr))) break;
+      // Z buffer -> g in GH (own tokens x 256 vocab) and GW (this / the peer CTA)
+      if (!(ok = mbar_wait(smem_u32(&zfull_bar), unit_it & 1u, abort_flag, a.err))) break;
+      tc_fence_after();
+      const uint32_t zaddr = tmem_base + lane_off + kZCol;
 #pragma unroll 1
       for (int c0 = 0; c0 < 256; c0 += 32) {
         float v[32];
-        tmem_ld32(taddr + c0, v);
+        tmem_ld32(zaddr + c0, v);
         uint32_t w[16];
         if (coef != 0.f) {
           const int lxc = lx - c0;
@@ -372,22 +370,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
       }
       fence_proxy_async_cluster();
-      release();
+      tc_fence_before();
       mbar_arrive_cluster(gready_leader);
-      // jobs dH: this CTA's 128 token rows x 256 columns of H
-      for (int nc = 0; nc < nC && ok; ++nc) {
-        if (!(ok = acquire_full(taddr))) break;
-        for (int c0 = 0; c0 < 256; c0 += 32)
-          drain_slab(&tm_dh, taddr + c0, nc * 256 + c0, own_row0 + q * 32, !own_null);
-        release();
+      // jobs: dH for 128 columns of H at a time, then dW
+      const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
+      for (int i = 0; i < nJ && ok; ++i) {
+        const uint32_t buf = jj & 1u, aph = (jj >> 1) & 1u;
+        if (!(ok = mbar_wait(smem_u32(&accf_bar[buf]), aph, abort_flag, a.err))) break;
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + lane_off + kAccCol + buf * 128;
+        if (i < nJH) {
+          for (int c0 = 0; c0 < 128; c0 += 32)
+            drain_slab(&tm_dh, taddr + c0, i * 128 + c0, own_row0 + q * 32, !own_null);
+        } else {
+          for (int c0 = 0; c0 < 128; c0 += 32)
+            drain_slab(&tm_dw, taddr + c0, (i - nJH) * 128 + c0, vrow, vrow < V);
+        }
+        tc_fence_before();
+        mbar_arrive_cluster(buf ? acce_leader1 : acce_leader0);
+        ++jj;
       }
-      // jobs dW: this CTA's 128 vocab rows x 256 columns of H
-      for (int nc = 0; nc < nC && ok; ++nc) {
-        if (!(ok = acquire_full(taddr))) break;
-        const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
-        for (int c0 = 0; c0 < 256; c0 += 32) drain_slab(&tm_dw, taddr + c0, nc * 256 + c0, vrow, vrow < V);
-        release();
-      }
+      ++unit_it;
     }
     if (lane == 0) bulk_wait_group<0>();
     __syncwarp();
