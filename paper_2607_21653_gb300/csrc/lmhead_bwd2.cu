@@ -386,8 +386,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           for (int c0 = 0; c0 < 128; c0 += 32)
             drain_slab(&tm_dw, taddr + c0, (i - nJH) * 128 + c0, vrow, vrow < V);
         }
+        // the accumulator was read with tcgen05.ld + wait::ld; a relaxed arrive
+        // after the tcgen05 fence is enough to hand it back to the MMA issuer
         tc_fence_before();
-        mbar_arrive_cluster(buf ? acce_leader1 : acce_leader0);
+        mbar_arrive_cluster_relaxed(buf ? acce_leader1 : acce_leader0);
         ++jj;
       }
       ++unit_it;
