@@ -206,6 +206,29 @@ def run_reference(args):
     return 0
 
 
+# ------------------------------------------------------------- multi-rank
+def rank_seed(workload_seed_default, rank, world):
+    """Seed of each rank's batch: the workload's own seed on a single GPU, a
+    distinct seed per rank otherwise (independent replicas, weak scaling)."""
+    return None if world == 1 else 2 + 100 * rank
+
+
+def max_over_ranks(value_ms, world, device=None):
+    """Slowest rank's time: every rank contributes its own elapsed time."""
+    if world == 1:
+        return float(value_ms)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value_ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank, world, steps, ms):
+    """Whole-job tokens/s: all ranks' tokens over the slowest rank's time."""
+    return world * tokens_per_rank * steps / (ms / 1e3)
+
+
 # ------------------------------------------------------------------ our arm
 def run_ours(args):
     import torch
@@ -225,7 +248,7 @@ def run_ours(args):
     molt.load()
     peaks = load_peaks()
 
-    w = make_workload(args.workload, seed=None if world == 1 else 2 + 100 * rank)
+    w = make_workload(args.workload, seed=rank_seed(None, rank, world))
     T, H, V = w.T, w.H, w.V
 
     def bf(bits):
@@ -285,10 +308,7 @@ def run_ours(args):
     timer.close()
     assert molt.device_status() == 0
     loss_val = float(out["loss"].item())
-    if world > 1:
-        tt = torch.tensor([ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
+    ms = max_over_ranks(ms, world, dev)
 
     # ---- end to end through the public API with host buffers
     e2e = None
@@ -319,11 +339,8 @@ def run_ours(args):
         e1.record()
         torch.cuda.synchronize()
         ems = e0.elapsed_time(e1)
-        if world > 1:
-            tt = torch.tensor([ems], dtype=torch.float64, device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            ems = float(tt.item())
-        e2e = {"value": world * T * e_steps / (ems / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+        ems = max_over_ranks(ems, world, dev)
+        e2e = {"value": job_throughput(T, world, e_steps, ems), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": 4, "steps": e_steps,
                "note": "hidden, tokens, mask, behaviour log-probs, rewards, group ids and the token->rollout map "
                        "copied from pinned host memory every step; W stays resident; loss read back"}
@@ -363,7 +380,7 @@ def run_ours(args):
 
     line = {
         "metric": METRIC,
-        "value": world * T * args.steps / (ms / 1e3),
+        "value": job_throughput(T, world, args.steps, ms),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
