@@ -94,6 +94,28 @@ molt_status molt_device_status(cudaStream_t stream, uint32_t* flags);
 molt_status molt_group_advantages(const float* rewards, const int32_t* group_ids, int64_t n_resp, double eps,
                                   float* adv_out, cudaStream_t stream);
 
+/* The advantage estimators Sec. 4.5 lists, per rollout (one reward each):
+ *   MOLT_ADV_GRPO          (r - mean_g) / (std_g + eps), unbiased std
+ *                          (identical to molt_group_advantages)
+ *   MOLT_ADV_GROUP_MEAN    r - mean_g (group-mean baseline)
+ *   MOLT_ADV_DR_GRPO       r - mean_g: Dr. GRPO drops the std division; its
+ *                          length normalisation is the token mean of Eq. 2
+ *   MOLT_ADV_RLOO          r_j - (sum_g r - r_j) / (n_g - 1) (leave-one-out)
+ *   MOLT_ADV_REINFORCE_PP  (r - mean_B) / (std_B + eps) over the whole batch;
+ *                          group_ids is ignored and may be NULL
+ * A group (or batch) of one response gives 0.  Same arithmetic contract as
+ * molt_group_advantages: fp64 in index order, bit-identical to a sequential
+ * fp64 evaluation rounded once to fp32. */
+typedef enum {
+  MOLT_ADV_GRPO = 0,
+  MOLT_ADV_GROUP_MEAN = 1,
+  MOLT_ADV_DR_GRPO = 2,
+  MOLT_ADV_RLOO = 3,
+  MOLT_ADV_REINFORCE_PP = 4
+} molt_adv_estimator;
+molt_status molt_advantages(const float* rewards, const int32_t* group_ids, int64_t n_resp, int estimator,
+                            double eps, float* adv_out, cudaStream_t stream);
+
 /* Per-token advantages: adv_tok[t] = adv_resp[resp_of_token[t]] (Sec. 4.2: the
  * rollout-level result is mapped back to its segments' tokens).
  * resp_of_token [T] int32 in [0, n_resp); out-of-range ids give 0. */

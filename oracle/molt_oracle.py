@@ -48,7 +48,7 @@ import math
 import numpy as np
 
 __all__ = [
-    "widen_bf16", "group_advantages", "broadcast_advantages", "logits_rows",
+    "widen_bf16", "group_advantages", "advantages", "ESTIMATORS", "broadcast_advantages", "logits_rows",
     "row_softmax_stats", "token_logprobs", "policy_loss", "policy_loss_rows",
     "clip_decision", "surrogate",
 ]
@@ -94,6 +94,73 @@ def group_advantages(rewards: np.ndarray, group_ids: np.ndarray,
             for j in range(start, end):
                 out[j] = np.float32((float(r[j]) - mean) / den)
         start = end
+    return out
+
+
+ESTIMATORS = ("grpo", "group_mean", "dr_grpo", "rloo", "reinforce_pp")
+
+
+def _runs(group_ids):
+    g = np.asarray(group_ids)
+    n = g.shape[0]
+    start = 0
+    while start < n:
+        end = start + 1
+        while end < n and g[end] == g[start]:
+            end += 1
+        yield start, end
+        start = end
+
+
+def advantages(rewards: np.ndarray, group_ids: np.ndarray, estimator: str = "grpo",
+               eps: float = DEFAULT_ADV_EPS) -> np.ndarray:
+    """The advantage estimators Sec. 4.5 lists, one reward per rollout (Sec. 4.2):
+
+    grpo          (r - mean_g) / (std_g + eps), unbiased std (see group_advantages)
+    group_mean    r - mean_g                           (group-mean baseline)
+    dr_grpo       r - mean_g  (Dr. GRPO drops the std division; its length
+                  normalisation is already the token-mean of Eq. 2)
+    rloo          r_j - (sum_g r - r_j) / (n_g - 1)    (leave-one-out baseline)
+    reinforce_pp  (r - mean_B) / (std_B + eps) over the whole batch B
+
+    Groups of one response (a batch of one for reinforce_pp) give 0.  fp64
+    sums in index order, one correctly rounded IEEE op at a time, one final
+    rounding to fp32."""
+    if estimator == "grpo":
+        return group_advantages(rewards, group_ids, eps)
+    r = np.asarray(rewards, dtype=np.float32)
+    n = r.shape[0]
+    out = np.zeros(n, dtype=np.float32)
+    if estimator == "reinforce_pp":
+        runs = [(0, n)] if n > 0 else []
+    elif estimator in ("group_mean", "dr_grpo", "rloo"):
+        runs = list(_runs(group_ids))
+    else:
+        raise ValueError(f"unknown estimator {estimator!r}")
+    for start, end in runs:
+        cnt = end - start
+        if cnt < 2:
+            continue
+        s = 0.0
+        for j in range(start, end):
+            s = s + float(r[j])
+        if estimator == "rloo":
+            for j in range(start, end):
+                baseline = (s - float(r[j])) / float(cnt - 1)
+                out[j] = np.float32(float(r[j]) - baseline)
+            continue
+        mean = s / float(cnt)
+        if estimator in ("group_mean", "dr_grpo"):
+            for j in range(start, end):
+                out[j] = np.float32(float(r[j]) - mean)
+            continue
+        ss = 0.0
+        for j in range(start, end):
+            d = float(r[j]) - mean
+            ss = ss + d * d
+        den = math.sqrt(ss / float(cnt - 1)) + eps
+        for j in range(start, end):
+            out[j] = np.float32((float(r[j]) - mean) / den)
     return out
 
 

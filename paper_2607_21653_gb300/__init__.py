@@ -110,6 +110,7 @@ def load():
         "molt_version": (I32, []),
         "molt_device_status": (I32, [P, ctypes.POINTER(ctypes.c_uint32)]),
         "molt_group_advantages": (I32, [P, P, I64, D, P, P]),
+        "molt_advantages": (I32, [P, P, I64, I32, D, P, P]),
         "molt_broadcast_advantages": (I32, [P, P, I64, I64, P, P]),
         "molt_mask_count": (I32, [P, I64, P, P]),
         "molt_token_logprobs_workspace_bytes": (SZ, [I64, I64, I64]),
@@ -257,6 +258,20 @@ def group_advantages(rewards, group_ids, eps: float = 1e-6, out=None, stream=Non
     out = torch.empty(n, dtype=torch.float32, device=rewards.device) if out is None else out
     _check(load().molt_group_advantages(_ptr(rewards, torch.float32, "rewards"), _ptr(group_ids, torch.int32, "group_ids"),
                                         n, float(eps), _ptr(out, torch.float32, "out"), _stream(stream)))
+    return out
+
+
+ESTIMATORS = {"grpo": 0, "group_mean": 1, "dr_grpo": 2, "rloo": 3, "reinforce_pp": 4}
+
+
+def advantages(rewards, group_ids, estimator="grpo", eps: float = 1e-6, out=None, stream=None):
+    """Per-rollout advantages with one of the estimators of Sec. 4.5."""
+    torch = _torch()
+    n = rewards.shape[0]
+    out = torch.empty(n, dtype=torch.float32, device=rewards.device) if out is None else out
+    gid = None if group_ids is None else _ptr(group_ids, torch.int32, "group_ids")
+    _check(load().molt_advantages(_ptr(rewards, torch.float32, "rewards"), gid, n, ESTIMATORS[estimator], float(eps),
+                                  _ptr(out, torch.float32, "out"), _stream(stream)))
     return out
 
 

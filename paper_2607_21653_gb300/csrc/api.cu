@@ -339,6 +339,24 @@ molt_status molt_group_advantages(const float* rewards, const int32_t* group_ids
   return MOLT_OK;
 }
 
+molt_status molt_advantages(const float* rewards, const int32_t* group_ids, int64_t n_resp, int estimator,
+                            double eps, float* adv_out, cudaStream_t stream) {
+  if (estimator < MOLT_ADV_GRPO || estimator > MOLT_ADV_REINFORCE_PP)
+    return fail(MOLT_ERR_INVALID_ARG, "unknown advantage estimator");
+  if (n_resp < 0 || n_resp >= (int64_t(1) << 26)) return fail(MOLT_ERR_INVALID_ARG, "n_resp out of range");
+  if (n_resp == 0) return MOLT_OK;
+  if (!rewards || !adv_out || (!group_ids && estimator != MOLT_ADV_REINFORCE_PP))
+    return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (!(eps >= 0.0)) return fail(MOLT_ERR_INVALID_ARG, "eps must be >= 0");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  MOLT_CUDA(launch_advantages(rewards, group_ids, static_cast<int>(n_resp), estimator, eps, adv_out, di->status,
+                              stream),
+            "advantages");
+  return MOLT_OK;
+}
+
 molt_status molt_broadcast_advantages(const float* adv_resp, const int32_t* resp_of_token, int64_t n_resp,
                                       int64_t T, float* adv_tok, cudaStream_t stream) {
   if (T < 0 || n_resp < 0 || T >= (int64_t(1) << 31) || n_resp >= (int64_t(1) << 31))

@@ -35,6 +35,9 @@ struct Workspace {
 };
 constexpr int kRedSlots = 8;
 
+// advantage estimators (values of molt_adv_estimator)
+constexpr int kAdvGrpo = 0, kAdvGroupMean = 1, kAdvDrGrpo = 2, kAdvRloo = 3, kAdvReinforcePP = 4;
+
 struct FwdArgs {
   const int32_t* tok_p;
   const int32_t* counts;
@@ -69,6 +72,8 @@ molt_status encode_tmap_2d(CUtensorMap* m, CUtensorMapDataType dt, int elem_byte
 // rows.cu
 cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
                                     unsigned* err, cudaStream_t s);
+cudaError_t launch_advantages(const float* rewards, const int32_t* gids, int n, int estimator, double eps,
+                              float* out, unsigned* err, cudaStream_t s);
 cudaError_t launch_broadcast(const float* adv, const int32_t* rot, int n_resp, int T, float* out, cudaStream_t s);
 cudaError_t launch_mask_count(const uint8_t* mask, int64_t T, int64_t* out, cudaStream_t s);
 cudaError_t launch_compact(const uint8_t* mask, int T, const Workspace& ws, cudaStream_t s);

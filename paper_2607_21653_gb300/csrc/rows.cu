@@ -14,37 +14,42 @@ namespace {
 constexpr float kLog2e = 1.4426950408889634f;
 
 // ---------------------------------------------------------------------------
-// GRPO advantages (Sec. 4.5 estimator list; Sec. 4.2 one reward per rollout).
-// One warp per response index; the warp whose index starts a run of equal ids
-// processes that group.  Lanes load the rewards coalesced, 32 at a time, and
-// lane 0 folds them with shuffles in index order, so the fp64 sums run in the
-// same order as a sequential loop.  Explicit _rn intrinsics keep the compiler
-// from contracting a multiply and an add into an FMA.
+// Advantage estimators (Sec. 4.5: GRPO, a group-mean baseline, Dr. GRPO, RLOO,
+// REINFORCE++; Sec. 4.2: one reward per rollout).  One warp per response index;
+// the warp whose index starts a run of equal ids processes that group (for
+// REINFORCE++, gid == nullptr and warp 0 normalises the whole batch).  Lanes
+// load the rewards coalesced, 32 at a time, and fold them with shuffles in
+// index order, so the fp64 sums run in the same order as a sequential loop.
+// Explicit _rn intrinsics keep the compiler from contracting a multiply and an
+// add into an FMA.
 // ---------------------------------------------------------------------------
 __global__ void group_adv_kernel(const float* __restrict__ r, const int32_t* __restrict__ gid, int n, double eps,
-                                 float* __restrict__ out, unsigned* err) {
+                                 int est, float* __restrict__ out, unsigned* err) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   if (warp >= n) return;
-  const int start = warp;
-  const int g = gid[start];
-  if (start > 0) {
-    const int gp = gid[start - 1];
-    if (gp == g) return;
-    if (gp > g && lane == 0) atomicOr(err, kDevErrUnsortedGroups);
-  }
-  // end of the run
-  int end = start;
-  for (int base = start;; base += 32) {
-    const int j = base + lane;
-    const bool same = (j < n) && (gid[j] == g);
-    const unsigned m = __ballot_sync(0xffffffffu, same);
-    if (m == 0xffffffffu) {
-      end = base + 32;
-      continue;
+  int start = warp, end = n;
+  if (gid == nullptr) {
+    if (warp != 0) return;
+  } else {
+    const int g = gid[start];
+    if (start > 0) {
+      const int gp = gid[start - 1];
+      if (gp == g) return;
+      if (gp > g && lane == 0) atomicOr(err, kDevErrUnsortedGroups);
     }
-    end = base + __ffs(~m) - 1;
-    break;
+    // end of the run
+    for (int base = start;; base += 32) {
+      const int j = base + lane;
+      const bool same = (j < n) && (gid[j] == g);
+      const unsigned m = __ballot_sync(0xffffffffu, same);
+      if (m == 0xffffffffu) {
+        end = base + 32;
+        continue;
+      }
+      end = base + __ffs(~m) - 1;
+      break;
+    }
   }
   const int cnt = end - start;
   if (cnt == 1) {
@@ -61,7 +66,27 @@ __global__ void group_adv_kernel(const float* __restrict__ r, const int32_t* __r
       s = __dadd_rn(s, vi);
     }
   }
-  const double mean = __ddiv_rn(__shfl_sync(0xffffffffu, s, 0), static_cast<double>(cnt));
+  s = __shfl_sync(0xffffffffu, s, 0);
+  if (est == kAdvRloo) {
+    // leave-one-out baseline (sum - r_j) / (n - 1)
+    for (int base = start; base < end; base += 32) {
+      const int j = base + lane;
+      if (j < end) {
+        const double rj = static_cast<double>(r[j]);
+        const double b = __ddiv_rn(__dsub_rn(s, rj), static_cast<double>(cnt - 1));
+        out[j] = __double2float_rn(__dsub_rn(rj, b));
+      }
+    }
+    return;
+  }
+  const double mean = __ddiv_rn(s, static_cast<double>(cnt));
+  if (est == kAdvGroupMean || est == kAdvDrGrpo) {
+    for (int base = start; base < end; base += 32) {
+      const int j = base + lane;
+      if (j < end) out[j] = __double2float_rn(__dsub_rn(static_cast<double>(r[j]), mean));
+    }
+    return;
+  }
   double ss = 0.0;
   for (int base = start; base < end; base += 32) {
     const int j = base + lane;
@@ -409,10 +434,22 @@ __global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __
 
 cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
                                     unsigned* err, cudaStream_t s) {
+  return launch_advantages(rewards, gids, n, kAdvGrpo, eps, out, err, s);
+}
+
+cudaError_t launch_advantages(const float* rewards, const int32_t* gids, int n, int estimator, double eps,
+                              float* out, unsigned* err, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
+  if (estimator == kAdvReinforcePP) {
+    // one warp over the whole batch; zero everything first so a batch of one gives 0
+    cudaError_t e = cudaMemsetAsync(out, 0, sizeof(float) * n, s);
+    if (e != cudaSuccess) return e;
+    group_adv_kernel<<<1, 32, 0, s>>>(rewards, nullptr, n, eps, estimator, out, err);
+    return cudaGetLastError();
+  }
   const int threads = 256;
   const int blocks = (int)(((int64_t)n * 32 + threads - 1) / threads);
-  group_adv_kernel<<<blocks, threads, 0, s>>>(rewards, gids, n, eps, out, err);
+  group_adv_kernel<<<blocks, threads, 0, s>>>(rewards, gids, n, eps, estimator, out, err);
   return cudaGetLastError();
 }
 

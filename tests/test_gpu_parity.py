@@ -53,6 +53,27 @@ def test_group_advantages_edge_cases():
     assert molt.device_status() & molt.DEV_FLAGS["unsorted_groups"]
 
 
+@pytest.mark.parametrize("estimator", ["grpo", "group_mean", "dr_grpo", "rloo", "reinforce_pp"])
+@pytest.mark.parametrize("name", ["tiny", "mid", "ragged"])
+def test_estimators_bit_exact(name, estimator):
+    w = make_workload(name, with_tensors=False)
+    ref = O.advantages(w.rewards, w.group_ids, estimator)
+    got = np_(molt.advantages(t(w.rewards), t(w.group_ids), estimator))
+    assert molt.device_status() == 0
+    np.testing.assert_array_equal(got.view(np.uint32), ref.view(np.uint32))
+
+
+def test_estimators_edge_cases():
+    r = np.array([1, 0, 0, 0, 5, 2, 2, 2, 7], np.float32)
+    g = np.array([0, 0, 0, 0, 1, 2, 2, 2, 3], np.int32)
+    for est in ("group_mean", "dr_grpo", "rloo", "reinforce_pp"):
+        got = np_(molt.advantages(t(r), t(g), est))
+        np.testing.assert_array_equal(got.view(np.uint32), O.advantages(r, g, est).view(np.uint32))
+    one = np.array([3.5], np.float32)
+    assert float(np_(molt.advantages(t(one), None, "reinforce_pp"))[0]) == 0.0
+    assert molt.device_status() == 0
+
+
 def test_broadcast_and_mask_count():
     w = make_workload("long_traj", with_tensors=False, T=8 * 1000)
     adv = O.group_advantages(w.rewards, w.group_ids)

@@ -268,3 +268,39 @@ def test_rows_subset_equals_full():
     for k in ("logp", "entropy", "ratio", "token_loss", "coef"):
         np.testing.assert_array_equal(sub[k], full[k][rows])
     np.testing.assert_allclose(sub["dH"], full["dH"][rows], rtol=1e-13, atol=1e-16)
+
+
+# ------------------------------------------------ other estimators (Sec. 4.5)
+def test_estimators_hand_values():
+    for row in _read_golden("estimators_hand.txt"):
+        est, rs, gs, want = [x.strip() for x in row.split("|")]
+        r = np.array([float(v) for v in rs.split()], dtype=np.float32)
+        g = np.array([int(v) for v in gs.split()], dtype=np.int32)
+        want = np.array([float(v) for v in want.split()], dtype=np.float64).astype(np.float32)
+        np.testing.assert_array_equal(O.advantages(r, g, est), want, err_msg=row)
+
+
+def test_estimators_match_numpy_and_relations():
+    rng = np.random.default_rng(21)
+    r = rng.random(48).astype(np.float32)
+    g = np.repeat(np.arange(6), 8).astype(np.int32)
+    r64 = r.astype(np.float64)
+    gm = O.advantages(r, g, "group_mean")
+    np.testing.assert_array_equal(gm, O.advantages(r, g, "dr_grpo"))
+    rloo = O.advantages(r, g, "rloo")
+    for k in range(6):
+        s = slice(8 * k, 8 * k + 8)
+        ref = r64[s] - r64[s].mean()
+        np.testing.assert_allclose(gm[s], ref.astype(np.float32), rtol=1e-6, atol=1e-7)
+        # leave-one-out = n/(n-1) times the group-mean baseline advantage
+        np.testing.assert_allclose(rloo[s], (8 / 7 * ref).astype(np.float32), rtol=2e-6, atol=1e-7)
+        # GRPO = group-mean advantage / (std + eps)
+        np.testing.assert_allclose(O.advantages(r, g, "grpo")[s], (ref / (r64[s].std(ddof=1) + 1e-6)).astype(np.float32),
+                                   rtol=2e-6, atol=1e-7)
+    rpp = O.advantages(r, g, "reinforce_pp")
+    np.testing.assert_allclose(rpp, ((r64 - r64.mean()) / (r64.std(ddof=1) + 1e-6)).astype(np.float32),
+                               rtol=2e-6, atol=1e-7)
+    assert abs(float(rpp.astype(np.float64).sum())) < 1e-4
+    # singleton groups and a batch of one give 0
+    assert (O.advantages(np.array([3.0], np.float32), np.array([0], np.int32), "rloo") == 0).all()
+    assert (O.advantages(np.array([3.0], np.float32), np.array([0], np.int32), "reinforce_pp") == 0).all()
