@@ -35,11 +35,24 @@ method at framework level only):
 * Backward: dL/dz_tv = (m_t / D) c_t (p_tv - [v == x_t]) with c_t = rho_t A_t on
   the unclipped branch and 0 on the clipped one; dH = G W, dW = G^T h.
 
+* Extended objective (policy_loss_ex; Sec. 4.5 names KL control and
+  rejection/weighting rules among the configurable pieces).  Readings: the KL
+  penalty to a reference policy is the per-token non-negative estimator
+  KL_t = e^r - r - 1 with r = ref_t - logp_t, weighted by kl_coef; the entropy
+  bonus subtracts entropy_coef * H_t and, unlike the reported entropy, carries
+  a gradient; the sequence gate rejects a whole sequence when the geometric
+  mean of its active tokens' ratios lies outside [gate_lo, gate_hi], setting
+  w_t = 0 for its tokens while D stays as given (Eq. 2 is not renormalised).
+  Per-row gradient: (m w / D)[(c + kl_coef(e^r - 1))(p - onehot)
+  + entropy_coef p (z - sum_v p_v z_v)].
+
 Pins (tests/test_oracle.py): closed-form advantages, zero/one-response groups,
 library log_softmax / entropy, sum exp(logp) = 1, the rho = 1 case against the
 autograd gradient of advantage-weighted cross-entropy, clipped rows having zero
 gradient, special clip values, finite differences of the loss, microbatch-split
-invariance of Eq. 2 and segment-split invariance of the advantages.
+invariance of Eq. 2 and segment-split invariance of the advantages; for the
+extended objective, torch autograd of PPO + k3 KL - entropy bonus, the
+reduction to the plain loss, and hand-built gate cases.
 """
 from __future__ import annotations
 
@@ -50,7 +63,7 @@ import numpy as np
 __all__ = [
     "widen_bf16", "group_advantages", "advantages", "ESTIMATORS", "broadcast_advantages", "logits_rows",
     "row_softmax_stats", "token_logprobs", "policy_loss", "policy_loss_rows",
-    "clip_decision", "surrogate",
+    "clip_decision", "surrogate", "policy_loss_ex", "sequence_gate",
 ]
 
 DEFAULT_ADV_EPS = 1e-6
@@ -313,3 +326,99 @@ def policy_loss(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, behavior_
     }
     r.update(loss=loss, denom=D, stats=stats)
     return r
+
+
+# --------------------------------------------------------------------------- #
+# Extended objective: KL to a reference policy, entropy bonus, sequence gate
+# --------------------------------------------------------------------------- #
+def sequence_gate(log_ratio: np.ndarray, seq: np.ndarray, mask: np.ndarray, lo: float, hi: float) -> np.ndarray:
+    """Per-token weight w_t in {0, 1} of a sequence-level importance gate
+    (Sec. 4.5: "a configurable rejection or weighting rule"; Sec. 4.3).
+    Reading: a sequence (maximal run of equal consecutive ids) is rejected when
+    the geometric mean of its active tokens' ratios, exp(mean_t (logp_t - b_t)),
+    lies outside [lo, hi]; all its tokens get w = 0.  fp64 sums in index order.
+    Tokens of sequences without active tokens keep w = 1 (they carry no loss)."""
+    lr = np.asarray(log_ratio, dtype=np.float64)
+    m = np.asarray(mask)
+    w = np.ones(lr.shape[0])
+    for start, end in _runs(seq):
+        s, n = 0.0, 0
+        for t in range(start, end):
+            if m[t]:
+                s = s + float(lr[t])
+                n += 1
+        if n == 0:
+            continue
+        g = math.exp(s / float(n))
+        if g < lo or g > hi:
+            w[start:end] = 0.0
+    return w
+
+
+def policy_loss_ex(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, behavior_logp: np.ndarray,
+                   adv: np.ndarray, mask: np.ndarray, eps_lo: float, eps_hi: float, denom: float | None = None,
+                   kl_coef: float = 0.0, ref_logp: np.ndarray | None = None, entropy_coef: float = 0.0,
+                   seq_of_token: np.ndarray | None = None, gate_lo: float = 0.0, gate_hi: float = float("inf"),
+                   block: int = 64):
+    """Full fp64 forward + backward of the extended per-token loss
+
+        l_t = w_t (l_pg,t + kl_coef KL_t - entropy_coef H_t),   L = sum_t m_t l_t / D
+
+    l_pg the clipped surrogate (see surrogate), KL_t = exp(r) - r - 1 with
+    r = ref_t - logp_t (the non-negative "k3" estimator of KL(pi || ref)), H_t
+    the token entropy, w_t the sequence-gate weight (1 without a gate).  D is
+    the Eq. 2 denominator (sum of the mask by default); rejected sequences do
+    not change it ("does not renormalize by the number of accepted sequences").
+    Gradient per row: (m w / D) [ (c + kl_coef (e^r - 1)) (p - onehot)
+                                  + entropy_coef p (z - sum_v p_v z_v) ]."""
+    T = hidden.shape[0]
+    m = np.asarray(mask).astype(np.float64)
+    D = float(m.sum()) if (denom is None or denom <= 0) else float(denom)
+    if D == 0.0:
+        raise ZeroDivisionError("Eq. 2 needs a nonzero denominator")
+    x_all = np.asarray(tokens)
+    b_all = np.asarray(behavior_logp, dtype=np.float64)
+    a_all = np.asarray(adv, dtype=np.float64)
+    # pass 1: log-probs of every active row (needed by the gate)
+    logp_all, ent_all = token_logprobs(hidden, W, x_all, mask, block=block)
+    w = np.ones(T)
+    if seq_of_token is not None:
+        w = sequence_gate(logp_all - b_all, seq_of_token, mask, gate_lo, gate_hi)
+    out = {k: np.zeros(T) for k in ("logp", "entropy", "ratio", "token_loss", "coef", "kl")}
+    out["clipped"] = np.zeros(T, dtype=bool)
+    out["gate"] = w
+    dH = np.zeros_like(hidden)
+    dW = np.zeros_like(W)
+    act = np.nonzero(m != 0)[0]
+    for b0 in range(0, act.shape[0], block):
+        t = act[b0:b0 + block]
+        z = logits_rows(hidden[t], W)
+        lse, logp, ent, p = row_softmax_stats(z, x_all[t])
+        rho = np.exp(logp - b_all[t])
+        l_pg, c, clipped = surrogate(rho, a_all[t], eps_lo, eps_hi)
+        if ref_logp is not None and kl_coef != 0.0:
+            r = np.asarray(ref_logp, dtype=np.float64)[t] - logp
+            kl = np.exp(r) - r - 1.0
+            c_kl = kl_coef * (np.exp(r) - 1.0)
+        else:
+            kl = np.zeros_like(logp)
+            c_kl = np.zeros_like(logp)
+        wt = w[t]
+        l_t = wt * (l_pg + kl_coef * kl - entropy_coef * ent)
+        coef = wt * (c + c_kl) / D
+        mu = (p * z).sum(axis=1)
+        g = coef[:, None] * p
+        g[np.arange(t.shape[0]), x_all[t]] -= coef
+        if entropy_coef != 0.0:
+            g += (wt * entropy_coef / D)[:, None] * p * (z - mu[:, None])
+        dH[t] = g @ W
+        dW += g.T @ hidden[t]
+        out["logp"][t] = logp
+        out["entropy"][t] = ent
+        out["ratio"][t] = rho
+        out["token_loss"][t] = l_t
+        out["coef"][t] = coef
+        out["kl"][t] = kl
+        out["clipped"][t] = clipped
+    out.update(loss=float(out["token_loss"].sum() / D), denom=D, dH=dH, dW=dW)
+    return out

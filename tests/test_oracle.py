@@ -304,3 +304,86 @@ def test_estimators_match_numpy_and_relations():
     # singleton groups and a batch of one give 0
     assert (O.advantages(np.array([3.0], np.float32), np.array([0], np.int32), "rloo") == 0).all()
     assert (O.advantages(np.array([3.0], np.float32), np.array([0], np.int32), "reinforce_pp") == 0).all()
+
+
+# ------------------------------------ extended objective (KL, entropy, gate)
+def _ex_problem(seed, T=12, H=10, V=24):
+    h, W, x, _ = _small_problem(seed, T=T, H=H, V=V)
+    rng = np.random.default_rng(seed + 100)
+    m = (rng.random(T) > 0.2).astype(np.uint8)
+    m[0] = 1
+    adv = rng.standard_normal(T)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    b = lp + rng.choice([-0.6, -0.1, 0.05, 0.4], size=T)
+    ref = lp + rng.normal(0, 0.3, T)
+    return h, W, x, m, adv, b, ref
+
+
+def test_ex_reduces_to_plain_loss():
+    h, W, x, m, adv, b, ref = _ex_problem(1)
+    plain = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.28)
+    ex = O.policy_loss_ex(h, W, x, b, adv, m, 0.2, 0.28)
+    np.testing.assert_allclose(ex["loss"], plain["loss"], rtol=1e-13)
+    np.testing.assert_allclose(ex["dH"], plain["dH"], rtol=1e-12, atol=1e-15)
+    np.testing.assert_allclose(ex["dW"], plain["dW"], rtol=1e-12, atol=1e-15)
+    # KL against the policy itself is zero and leaves the gradient unchanged
+    lp, _ = O.token_logprobs(h, W, x, None)
+    ex0 = O.policy_loss_ex(h, W, x, b, adv, m, 0.2, 0.28, kl_coef=0.7, ref_logp=lp)
+    np.testing.assert_allclose(ex0["kl"], 0.0, atol=1e-12)
+    np.testing.assert_allclose(ex0["dH"], plain["dH"], rtol=1e-9, atol=1e-14)
+
+
+def test_ex_gradient_matches_autograd():
+    """Independent derivation: torch autograd of PPO + k3 KL - entropy bonus."""
+    torch = pytest.importorskip("torch")
+    h, W, x, m, adv, b, ref = _ex_problem(2)
+    kl_c, ent_c, D = 0.3, 0.05, 11.0
+    r = O.policy_loss_ex(h, W, x, b, adv, m, 0.2, 0.28, denom=D, kl_coef=kl_c, ref_logp=ref, entropy_coef=ent_c)
+    th = torch.tensor(h, requires_grad=True)
+    tW = torch.tensor(W, requires_grad=True)
+    logits = th @ tW.T
+    logsm = torch.log_softmax(logits, dim=1)
+    logp = logsm[torch.arange(len(x)), torch.tensor(x)]
+    ent = -(logsm.exp() * logsm).sum(dim=1)
+    rho = torch.exp(logp - torch.tensor(b))
+    A = torch.tensor(adv)
+    pg = -torch.minimum(rho * A, torch.clamp(rho, 0.8, 1.28) * A)
+    rr = torch.tensor(ref) - logp
+    kl = torch.exp(rr) - rr - 1
+    L = (torch.tensor(m, dtype=torch.float64) * (pg + kl_c * kl - ent_c * ent)).sum() / D
+    L.backward()
+    np.testing.assert_allclose(r["loss"], L.item(), rtol=1e-12)
+    np.testing.assert_allclose(r["dH"], th.grad.numpy(), rtol=1e-9, atol=1e-13)
+    np.testing.assert_allclose(r["dW"], tW.grad.numpy(), rtol=1e-9, atol=1e-13)
+
+
+def test_sequence_gate_rejects_without_renormalising():
+    """Sec. 4.5: rejection weights live in l_i; Eq. 2 keeps its denominator."""
+    h, W, x, _ = _small_problem(3, T=12, H=8, V=16)
+    m = np.ones(12, np.uint8)
+    adv = np.random.default_rng(3).standard_normal(12)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    seq = np.repeat(np.arange(3), 4).astype(np.int32)
+    # per-sequence log ratios: seq 0 all +0.1 (ratio 1.105, kept), seq 1 mean +0.6
+    # (ratio 1.82, rejected above 1.5), seq 2 mean -1.0 (ratio 0.37, rejected below 0.5)
+    lr = np.array([0.1] * 4 + [0.9, 0.3, 0.6, 0.6] + [-1.0, -1.2, -0.8, -1.0])
+    b = lp - lr
+    w = O.sequence_gate(lr, seq, m, 0.5, 1.5)
+    np.testing.assert_array_equal(w, [1] * 4 + [0] * 8)
+    ex = O.policy_loss_ex(h, W, x, b, adv, m, 0.2, 0.2, seq_of_token=seq, gate_lo=0.5, gate_hi=1.5)
+    plain = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.2)
+    assert ex["denom"] == 12.0
+    np.testing.assert_allclose(ex["token_loss"][:4], plain["token_loss"][:4], rtol=1e-13)
+    assert (ex["token_loss"][4:] == 0).all() and (ex["dH"][4:] == 0).all()
+    np.testing.assert_allclose(ex["loss"], plain["token_loss"][:4].sum() / 12.0, rtol=1e-13)
+    # masked tokens do not enter the geometric mean
+    m2 = m.copy()
+    m2[4] = 0
+    # with hi = 1.7: seq 1 with all four tokens has ratio e^0.6 = 1.82 (rejected);
+    # without its masked 0.9 token the mean is 0.5, ratio 1.65 (kept)
+    np.testing.assert_array_equal(O.sequence_gate(lr, seq, m, 0.5, 1.7)[4:8], 0.0)
+    np.testing.assert_array_equal(O.sequence_gate(lr, seq, m2, 0.5, 1.7)[4:8], 1.0)
+    # a sequence with no active token keeps weight 1 and contributes nothing
+    m3 = m.copy()
+    m3[8:] = 0
+    np.testing.assert_array_equal(O.sequence_gate(lr, seq, m3, 0.5, 1.5)[8:], 1.0)
