@@ -178,6 +178,61 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
                                      size_t workspace_bytes, cudaStream_t stream);
 
 /*
+ * Extended objective (Sec. 4.5 lists KL control and rejection / weighting rules
+ * among the configurable parts of the policy update).  Per active token t:
+ *   l_t = w_t (l_pg,t + kl_coef KL_t - entropy_coef H_t)
+ *   KL_t = exp(r_t) - r_t - 1,  r_t = ref_logp[t] - logp_t   (non-negative
+ *          per-token estimator of KL(pi || pi_ref))
+ *   H_t  = entropy of softmax(z_t); the bonus carries a gradient
+ *   w_t  = sequence-gate weight in {0, 1}: a sequence is rejected (w = 0 on all
+ *          its tokens) when the geometric mean of its active tokens' ratios,
+ *          exp(mean_t (logp_t - behavior_logp[t])), lies outside
+ *          [gate_lo, gate_hi].  D is not renormalised by the rejections (Eq. 2).
+ *   dL/dz_tv = (m_t w_t / D) [ (c_t + kl_coef (exp(r_t) - 1)) (p_tv - [v == x_t])
+ *                             + entropy_coef p_tv (z_tv - sum_u p_tu z_tu) ]
+ * Fields:
+ *   kl_coef       >= 0; 0 disables the KL term (ref_logp may then be NULL)
+ *   entropy_coef  finite; 0 disables the bonus and its gradient
+ *   ref_logp      [T] device fp32, reference-policy log-prob of tokens[t]
+ *   seq_of_token  [T] device int32 sequence ids, non-decreasing (a sequence is
+ *                 the run of tokens sharing an id); NULL disables the gate.
+ *                 Decreasing ids set MOLT_DEV_UNSORTED_GROUPS.
+ *   gate_lo, gate_hi   acceptance band of the geometric-mean ratio,
+ *                 0 <= gate_lo <= gate_hi (gate_hi may be +inf)
+ */
+typedef struct {
+  float kl_coef;
+  float entropy_coef;
+  const float* ref_logp;
+  const int32_t* seq_of_token;
+  double gate_lo;
+  double gate_hi;
+} molt_loss_options;
+
+/* molt_stats plus the extended objective's counters (device memory). */
+typedef struct {
+  molt_stats base;           /* as above; n_clip_* count accepted tokens only */
+  double sum_kl;             /* sum of KL_t over accepted active tokens */
+  int64_t n_tokens_rejected; /* active tokens of rejected sequences */
+  int64_t n_seq_rejected;    /* sequences (with at least one active token) rejected */
+} molt_stats_ex;
+
+/*
+ * molt_policy_loss_fwd_bwd with the extended objective above.  Arguments as in
+ * molt_policy_loss_fwd_bwd; opts NULL (or all terms disabled) gives the same
+ * results.  token_loss_out[t] = m_t l_t with the extended l_t.  The workspace
+ * size is molt_policy_loss_workspace_bytes(T, H, V).
+ */
+molt_status molt_policy_loss_fwd_bwd_ex(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                                        const float* behavior_logp, const float* adv, const uint8_t* mask,
+                                        int64_t T, int64_t H, int64_t V, float clip_lo, float clip_hi,
+                                        double denom, const molt_loss_options* opts, float* loss_out,
+                                        uint16_t* dhidden_out, float* dW_out, int accumulate_dW,
+                                        float* logp_out, float* entropy_out, float* token_loss_out,
+                                        molt_stats_ex* stats_out, void* workspace, size_t workspace_bytes,
+                                        cudaStream_t stream);
+
+/*
  * Allocation-free variant of molt_token_logprobs_fwd (the paper has no
  * counterpart; it exists for callers, not for the method).
  *

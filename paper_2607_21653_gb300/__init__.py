@@ -118,6 +118,8 @@ def load():
         "molt_policy_loss_workspace_bytes": (SZ, [I64, I64, I64]),
         "molt_policy_loss_fwd_bwd": (I32, [P, P, P, P, P, P, I64, I64, I64, F, F, D, P, P, P, I32, P, P, P, P,
                                             P, SZ, P]),
+        "molt_policy_loss_fwd_bwd_ex": (I32, [P, P, P, P, P, P, I64, I64, I64, F, F, D, P, P, P, P, I32, P, P,
+                                               P, P, P, SZ, P]),
         "molt_set_timing_events": (None, [P, P, I32]),
         "molt_token_logprobs_fwd_noalloc": (I32, [P, P, P, P, I64, I64, I64, P, P, P]),
     }
@@ -379,11 +381,60 @@ def policy_loss_fwd_bwd(hidden, weight, tokens, behavior_logp, adv, mask=None, c
 
 
 def stats_dict(stats_tensor) -> dict:
-    """Decode the molt_stats struct (5 doubles + 3 int64) copied to the host."""
+    """Decode molt_stats (5 doubles + 3 int64) or molt_stats_ex (those, then
+    1 double + 2 int64) copied to the host."""
     import numpy as np
     raw = stats_tensor.detach().cpu().numpy().view(np.uint8).tobytes()
     d = np.frombuffer(raw[:40], dtype=np.float64)
     i = np.frombuffer(raw[40:64], dtype=np.int64)
-    return {"denom": float(d[0]), "loss": float(d[1]), "sum_ratio": float(d[2]), "sum_entropy": float(d[3]),
-            "max_abs_log_ratio": float(d[4]), "n_active": int(i[0]), "n_clip_low": int(i[1]),
-            "n_clip_high": int(i[2])}
+    out = {"denom": float(d[0]), "loss": float(d[1]), "sum_ratio": float(d[2]), "sum_entropy": float(d[3]),
+           "max_abs_log_ratio": float(d[4]), "n_active": int(i[0]), "n_clip_low": int(i[1]),
+           "n_clip_high": int(i[2])}
+    if len(raw) >= 88:
+        out["sum_kl"] = float(np.frombuffer(raw[64:72], dtype=np.float64)[0])
+        j = np.frombuffer(raw[72:88], dtype=np.int64)
+        out["n_tokens_rejected"] = int(j[0])
+        out["n_seq_rejected"] = int(j[1])
+    return out
+
+
+class LossOptions(ctypes.Structure):
+    """molt_loss_options: KL-to-reference, entropy bonus, sequence gate."""
+    _fields_ = [("kl_coef", ctypes.c_float), ("entropy_coef", ctypes.c_float), ("ref_logp", ctypes.c_void_p),
+                ("seq_of_token", ctypes.c_void_p), ("gate_lo", ctypes.c_double), ("gate_hi", ctypes.c_double)]
+
+
+def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None, clip_lo=0.2, clip_hi=0.2,
+                           denom=0.0, kl_coef=0.0, ref_logp=None, entropy_coef=0.0, seq_of_token=None,
+                           gate_lo=0.0, gate_hi=float("inf"), dW=None, accumulate_dW=False,
+                           want_token_outputs=True, stream=None, workspace=None):
+    """policy_loss_fwd_bwd with the extended objective
+    l_t = w_t (l_pg,t + kl_coef KL_t - entropy_coef H_t) (molt_policy_loss_fwd_bwd_ex).
+    Returns the same dict; stats is molt_stats_ex (11 x 8 bytes)."""
+    torch = _torch()
+    T, H = hidden.shape
+    V = weight.shape[0]
+    dev = hidden.device
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    dh = torch.empty(T, H, dtype=torch.bfloat16, device=dev)
+    if dW is None:
+        dW = torch.empty(V, H, dtype=torch.float32, device=dev)
+        accumulate_dW = False
+    stats = torch.zeros(11, dtype=torch.float64, device=dev)
+    logp = ent = tl = None
+    if want_token_outputs:
+        logp = torch.empty(T, dtype=torch.float32, device=dev)
+        ent = torch.empty(T, dtype=torch.float32, device=dev)
+        tl = torch.empty(T, dtype=torch.float32, device=dev)
+    opts = LossOptions(float(kl_coef), float(entropy_coef), _ptr(ref_logp, torch.float32, "ref_logp"),
+                       _ptr(seq_of_token, torch.int32, "seq_of_token"), float(gate_lo), float(gate_hi))
+    nbytes = policy_loss_workspace_bytes(T, H, V)
+    ws = workspace if workspace is not None else _workspace(nbytes, dev, "policy_loss")
+    _check(load().molt_policy_loss_fwd_bwd_ex(
+        _bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"), _ptr(tokens, torch.int32, "tokens"),
+        _ptr(behavior_logp, torch.float32, "behavior_logp"), _ptr(adv, torch.float32, "adv"),
+        _ptr(mask, torch.uint8, "mask"), T, H, V, float(clip_lo), float(clip_hi), float(denom),
+        ctypes.byref(opts), _ptr(loss), _ptr(dh), _ptr(dW, torch.float32, "dW"), 1 if accumulate_dW else 0,
+        _ptr(logp), _ptr(ent), _ptr(tl), _ptr(stats), ws.data_ptr(), ws.numel(), _stream(stream)))
+    return {"loss": loss, "dhidden": dh, "dW": dW, "logp": logp, "entropy": ent, "token_loss": tl,
+            "stats": stats}

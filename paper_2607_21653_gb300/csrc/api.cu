@@ -124,7 +124,8 @@ int choose_splits(int64_t Tcap, int64_t V, int n_sm) {
 }
 
 struct Layout {
-  size_t counts, row_map, pos, tok_p, b_p, adv_p, h_p, part, zx, lse, coef, tile_flag, tile_list, red, dh32, total;
+  size_t counts, row_map, pos, tok_p, b_p, adv_p, h_p, part, zx, lse, coef, tile_flag, tile_list, red, dh32;
+  size_t lp_p, ent_p, ecoef, mu, gate_p, total;
 };
 
 Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd) {
@@ -152,6 +153,11 @@ Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd) {
   L.tile_list = take(ntile * 4);
   L.red = take(ntile * kRedSlots * 8);
   L.dh32 = with_bwd ? take(Tcap * H * 4) : o;
+  L.lp_p = with_bwd ? take(Tcap * 4) : o;
+  L.ent_p = with_bwd ? take(Tcap * 4) : o;
+  L.ecoef = with_bwd ? take(Tcap * 4) : o;
+  L.mu = with_bwd ? take(Tcap * 4) : o;
+  L.gate_p = with_bwd ? take(Tcap) : o;
   L.total = o + 256;   // slack for aligning the caller's base pointer
   (void)V;
   return L;
@@ -175,6 +181,11 @@ Workspace carve(void* base, const Layout& L) {
   w.tile_list = reinterpret_cast<int32_t*>(p + L.tile_list);
   w.red = reinterpret_cast<double*>(p + L.red);
   w.dh32 = reinterpret_cast<float*>(p + L.dh32);
+  w.lp_p = reinterpret_cast<float*>(p + L.lp_p);
+  w.ent_p = reinterpret_cast<float*>(p + L.ent_p);
+  w.ecoef = reinterpret_cast<float*>(p + L.ecoef);
+  w.mu = reinterpret_cast<float*>(p + L.mu);
+  w.gate_p = p + L.gate_p;
   return w;
 }
 
@@ -253,6 +264,114 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
   ev_start(1, s);
   MOLT_CUDA(launch_lmhead_fwd(tm_h, tm_w, fa, di->n_sm, s), "lmhead forward");
   ev_stop(1, s);
+  return MOLT_OK;
+}
+
+// Both loss entry points.  opts == nullptr runs the plain clipped surrogate
+// (one merge kernel computes the loss rows); otherwise the merge only writes
+// the packed log-probs and entropies, the sequence gate runs on them, and a
+// second row kernel forms the extended loss and the backward coefficients.
+molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                             const float* behavior_logp, const float* adv, const uint8_t* mask, int64_t T,
+                             int64_t H, int64_t V, float clip_lo, float clip_hi, double denom,
+                             const molt_loss_options* opts, float* loss_out, uint16_t* dhidden_out, float* dW_out,
+                             int accumulate_dW, float* logp_out, float* entropy_out, float* token_loss_out,
+                             molt_stats* stats_out, molt_stats_ex* stats_ex_out, void* workspace,
+                             size_t workspace_bytes, cudaStream_t stream) {
+  MOLT_TRY(check_shape(T, H, V));
+  if (!hidden || !W || !tokens || !behavior_logp || !adv || !loss_out || !dhidden_out || !dW_out)
+    return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(hidden) || !aligned16(W) || !aligned16(dhidden_out) || !aligned16(dW_out))
+    return fail(MOLT_ERR_INVALID_ARG, "hidden, W, dhidden and dW must be 16-byte aligned");
+  if (!(clip_lo >= 0.f && clip_lo < 1.f) || !(clip_hi >= 0.f) || clip_hi != clip_hi || clip_hi > 1e30f)
+    return fail(MOLT_ERR_INVALID_ARG, "clip bounds must satisfy 0 <= clip_lo < 1 and clip_hi >= 0");
+  if (denom != denom) return fail(MOLT_ERR_INVALID_ARG, "denom is NaN");
+  LossEx ex{};
+  if (opts) {
+    ex.kl_coef = opts->kl_coef;
+    ex.entropy_coef = opts->entropy_coef;
+    ex.ref_logp = opts->ref_logp;
+    ex.seq = opts->seq_of_token;
+    ex.gate_lo = opts->gate_lo;
+    ex.gate_hi = opts->gate_hi;
+    if (!(ex.kl_coef >= 0.f) || ex.kl_coef > 1e30f) return fail(MOLT_ERR_INVALID_ARG, "kl_coef must be finite and >= 0");
+    if (ex.kl_coef != 0.f && !ex.ref_logp) return fail(MOLT_ERR_INVALID_ARG, "kl_coef > 0 needs ref_logp");
+    if (!(ex.entropy_coef >= -1e30f && ex.entropy_coef <= 1e30f))
+      return fail(MOLT_ERR_INVALID_ARG, "entropy_coef must be finite");
+    if (ex.seq && !(ex.gate_lo >= 0.0 && ex.gate_hi >= ex.gate_lo))
+      return fail(MOLT_ERR_INVALID_ARG, "the gate band must satisfy 0 <= gate_lo <= gate_hi");
+  }
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  if (T == 0) {
+    // nothing to compute: loss 0, stats zero, dW untouched or zeroed
+    MOLT_CUDA(cudaMemsetAsync(loss_out, 0, sizeof(float), stream), "memset loss");
+    if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, V * H * sizeof(float), stream), "memset dW");
+    if (stats_out) MOLT_CUDA(cudaMemsetAsync(stats_out, 0, sizeof(molt_stats), stream), "memset stats");
+    if (stats_ex_out) MOLT_CUDA(cudaMemsetAsync(stats_ex_out, 0, sizeof(molt_stats_ex), stream), "memset stats");
+    return MOLT_OK;
+  }
+  const int64_t Tcap = round_tiles(T);
+  const int S = choose_splits(Tcap, V, di->n_sm);
+  const Layout L = layout(T, H, V, S, true);
+  Scratch sc;
+  MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
+  const Workspace w = carve(sc.ptr, L);
+  const bool pair_bwd = (H % 256) == 0;
+  CUtensorMap tm_h, tm_w, tm_wz, tm_wn, tm_dh, tm_dw;
+  MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
+  MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
+  MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, pair_bwd ? 128 : kBwdBV));
+  MOLT_TRY(make_tmap(&tm_wn, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, 64));
+  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
+  MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
+  MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
+  if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
+  if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
+  if (token_loss_out) MOLT_CUDA(cudaMemsetAsync(token_loss_out, 0, T * sizeof(float), stream), "memset token loss");
+  ev_start(2, stream);
+  if (opts) {
+    MOLT_CUDA(launch_merge_stats_ex(static_cast<int>(Tcap), static_cast<int>(V), S, w, logp_out, entropy_out,
+                                    di->status, stream),
+              "merge");
+    MOLT_CUDA(launch_seq_gate(static_cast<int>(T), static_cast<int>(Tcap), ex, w, di->status, stream), "gate");
+    MOLT_CUDA(launch_loss_rows_ex(static_cast<int>(Tcap), denom, clip_lo, clip_hi, ex, w, token_loss_out, stream),
+              "loss rows");
+  } else {
+    MOLT_CUDA(launch_merge(true, static_cast<int>(Tcap), static_cast<int>(V), S, denom, clip_lo, clip_hi, w,
+                           logp_out, entropy_out, token_loss_out, di->status, stream),
+              "merge");
+  }
+  MOLT_CUDA(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, stats_ex_out, di->status, stream),
+            "finalize");
+  ev_stop(2, stream);
+  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
+  if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
+  BwdArgs ba{};
+  ba.tok_p = w.tok_p;
+  ba.lse = w.lse;
+  ba.coef = w.coef;
+  ba.counts = w.counts;
+  ba.tile_list = w.tile_list;
+  ba.V = static_cast<int>(V);
+  ba.H = static_cast<int>(H);
+  ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
+  ba.tile_group = pair_bwd ? 8 : 16;
+  if (opts && ex.entropy_coef != 0.f) {
+    ba.ecoef = w.ecoef;
+    ba.mu = w.mu;
+  }
+  ba.err = di->status;
+  ev_start(3, stream);
+  if (pair_bwd)
+    MOLT_CUDA(launch_lmhead_bwd_pair(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  else
+    MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  ev_stop(3, stream);
+  ev_start(4, stream);
+  MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
+  ev_stop(4, stream);
   return MOLT_OK;
 }
 
@@ -433,71 +552,24 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
                                      int accumulate_dW, float* logp_out, float* entropy_out,
                                      float* token_loss_out, molt_stats* stats_out, void* workspace,
                                      size_t workspace_bytes, cudaStream_t stream) {
-  MOLT_TRY(check_shape(T, H, V));
-  if (!hidden || !W || !tokens || !behavior_logp || !adv || !loss_out || !dhidden_out || !dW_out)
-    return fail(MOLT_ERR_INVALID_ARG, "null pointer");
-  if (!aligned16(hidden) || !aligned16(W) || !aligned16(dhidden_out) || !aligned16(dW_out))
-    return fail(MOLT_ERR_INVALID_ARG, "hidden, W, dhidden and dW must be 16-byte aligned");
-  if (!(clip_lo >= 0.f && clip_lo < 1.f) || !(clip_hi >= 0.f) || clip_hi != clip_hi || clip_hi > 1e30f)
-    return fail(MOLT_ERR_INVALID_ARG, "clip bounds must satisfy 0 <= clip_lo < 1 and clip_hi >= 0");
-  if (denom != denom) return fail(MOLT_ERR_INVALID_ARG, "denom is NaN");
-  molt_status st;
-  const DeviceInfo* di = device_info(&st);
-  if (!di) return st;
-  if (T == 0) {
-    // nothing to compute: loss 0, stats zero, dW untouched or zeroed
-    MOLT_CUDA(cudaMemsetAsync(loss_out, 0, sizeof(float), stream), "memset loss");
-    if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, V * H * sizeof(float), stream), "memset dW");
-    if (stats_out) MOLT_CUDA(cudaMemsetAsync(stats_out, 0, sizeof(molt_stats), stream), "memset stats");
-    return MOLT_OK;
-  }
-  const int64_t Tcap = round_tiles(T);
-  const int S = choose_splits(Tcap, V, di->n_sm);
-  const Layout L = layout(T, H, V, S, true);
-  Scratch sc;
-  MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
-  const Workspace w = carve(sc.ptr, L);
-  const bool pair_bwd = (H % 256) == 0;
-  CUtensorMap tm_h, tm_w, tm_wz, tm_wn, tm_dh, tm_dw;
-  MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
-  MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
-  MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, pair_bwd ? 128 : kBwdBV));
-  MOLT_TRY(make_tmap(&tm_wn, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, 64));
-  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
-  MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
-  MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
-  if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
-  if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
-  if (token_loss_out) MOLT_CUDA(cudaMemsetAsync(token_loss_out, 0, T * sizeof(float), stream), "memset token loss");
-  ev_start(2, stream);
-  MOLT_CUDA(launch_merge(true, static_cast<int>(Tcap), static_cast<int>(V), S, denom, clip_lo, clip_hi, w, logp_out,
-                         entropy_out, token_loss_out, di->status, stream),
-            "merge");
-  MOLT_CUDA(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, di->status, stream), "finalize");
-  ev_stop(2, stream);
-  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
-  if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
-  BwdArgs ba{};
-  ba.tok_p = w.tok_p;
-  ba.lse = w.lse;
-  ba.coef = w.coef;
-  ba.counts = w.counts;
-  ba.tile_list = w.tile_list;
-  ba.V = static_cast<int>(V);
-  ba.H = static_cast<int>(H);
-  ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
-  ba.tile_group = pair_bwd ? 8 : 16;
-  ba.err = di->status;
-  ev_start(3, stream);
-  if (pair_bwd)
-    MOLT_CUDA(launch_lmhead_bwd_pair(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
-  else
-    MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
-  ev_stop(3, stream);
-  ev_start(4, stream);
-  MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
-  ev_stop(4, stream);
-  return MOLT_OK;
+  return policy_loss_impl(hidden, W, tokens, behavior_logp, adv, mask, T, H, V, clip_lo, clip_hi, denom, nullptr,
+                          loss_out, dhidden_out, dW_out, accumulate_dW, logp_out, entropy_out, token_loss_out,
+                          stats_out, nullptr, workspace, workspace_bytes, stream);
+}
+
+molt_status molt_policy_loss_fwd_bwd_ex(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
+                                        const float* behavior_logp, const float* adv, const uint8_t* mask,
+                                        int64_t T, int64_t H, int64_t V, float clip_lo, float clip_hi,
+                                        double denom, const molt_loss_options* opts, float* loss_out,
+                                        uint16_t* dhidden_out, float* dW_out, int accumulate_dW,
+                                        float* logp_out, float* entropy_out, float* token_loss_out,
+                                        molt_stats_ex* stats_out, void* workspace, size_t workspace_bytes,
+                                        cudaStream_t stream) {
+  molt_loss_options none{};
+  none.gate_hi = 0.0;
+  return policy_loss_impl(hidden, W, tokens, behavior_logp, adv, mask, T, H, V, clip_lo, clip_hi, denom,
+                          opts ? opts : &none, loss_out, dhidden_out, dW_out, accumulate_dW, logp_out, entropy_out,
+                          token_loss_out, nullptr, stats_out, workspace, workspace_bytes, stream);
 }
 
 }  // extern "C"

@@ -1,6 +1,7 @@
 // Backward pass of the fused LM-head + clipped-surrogate loss (Sec. 4.5, Eq. 2).
 //
 //   g_tv = coef_t (softmax(z_t)_v - [v == x_t]),  coef_t = m_t c_t / D
+//          (+ ecoef_t softmax(z_t)_v (z_tv - mu_t) with an entropy bonus)
 //   dH_t = sum_v g_tv W_v          dW_v = sum_t g_tv h_t
 //
 // Neither the logits nor g touch global memory.  A work unit is one 128-row
@@ -70,6 +71,7 @@ __device__ __forceinline__ void write_box(uint32_t box, int lane, const float (&
   }
 }
 
+template <bool kEnt>
 __global__ void __launch_bounds__(kThreads, 1)
     lmhead_bwd_kernel(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_wz,
                       const __grid_constant__ CUtensorMap tm_wn, const __grid_constant__ CUtensorMap tm_dh,
@@ -292,7 +294,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int n_mh = (V - v0 > 128) ? 2 : 1;
       const int row = row0 + r;
       const float coef = a.coef[row];
-      const float lseL = (coef != 0.f) ? a.lse[row] * kLog2e : 0.f;
+      float ecoef = 0.f, mu = 0.f;
+      if constexpr (kEnt) {
+        ecoef = a.ecoef[row];
+        mu = a.mu[row];
+      }
+      const bool live = kEnt ? (coef != 0.f || ecoef != 0.f) : (coef != 0.f);
+      const float lseL = live ? a.lse[row] * kLog2e : 0.f;
       const int lx = a.tok_p[row] - v0;
       uint32_t taddr;
       // job Z -> g in shared memory
@@ -302,13 +310,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         float v[32];
         tmem_ld32(taddr + c0, v);
         uint32_t w[16];
-        if (coef != 0.f) {
+        if (live) {
           const int lxc = lx - c0;
           const int nvalid = V - v0 - c0;
 #pragma unroll
           for (int j = 0; j < 32; j += 2) {
-            float g0 = coef * ex2_approx(fmaf(v[j], kLog2e, -lseL));
-            float g1 = coef * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+            float g0, g1;
+            if constexpr (kEnt) {   // p (coef + ecoef (z - mu)): the entropy-bonus term
+              g0 = fmaf(ecoef, v[j] - mu, coef) * ex2_approx(fmaf(v[j], kLog2e, -lseL));
+              g1 = fmaf(ecoef, v[j + 1] - mu, coef) * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+            } else {
+              g0 = coef * ex2_approx(fmaf(v[j], kLog2e, -lseL));
+              g1 = coef * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+            }
             if (j == lxc) g0 -= coef;
             if (j + 1 == lxc) g1 -= coef;
             if (j >= nvalid) g0 = 0.f;
@@ -367,9 +381,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 cudaError_t launch_lmhead_bwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w_z, const CUtensorMap& tm_w_n,
                               const CUtensorMap& tm_dh, const CUtensorMap& tm_dw, const BwdArgs& a, int grid,
                               cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(lmhead_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  const bool ent = a.ecoef != nullptr;
+  cudaError_t e = ent ? cudaFuncSetAttribute(lmhead_bwd_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSmemBytes)
+                      : cudaFuncSetAttribute(lmhead_bwd_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSmemBytes);
   if (e != cudaSuccess) return e;
-  lmhead_bwd_kernel<<<grid, kThreads, kSmemBytes, s>>>(tm_h, tm_w_z, tm_w_n, tm_dh, tm_dw, a);
+  if (ent)
+    lmhead_bwd_kernel<true><<<grid, kThreads, kSmemBytes, s>>>(tm_h, tm_w_z, tm_w_n, tm_dh, tm_dw, a);
+  else
+    lmhead_bwd_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(tm_h, tm_w_z, tm_w_n, tm_dh, tm_dw, a);
   return cudaGetLastError();
 }
 

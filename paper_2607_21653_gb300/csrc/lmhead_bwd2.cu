@@ -2,6 +2,7 @@
 // (tcgen05 cta_group::2), used when H is a multiple of 256.
 //
 //   g_tv = coef_t (softmax(z_t)_v - [v == x_t]),  coef_t = m_t c_t / D   (Eq. 2)
+//          (+ ecoef_t softmax(z_t)_v (z_tv - mu_t) with an entropy bonus)
 //   dH_t = sum_v g_tv W_v          dW_v = sum_t g_tv h_t
 //
 // A pair unit is 256 active token rows (two 128-row tiles, one per CTA) times a
@@ -92,6 +93,7 @@ __device__ __forceinline__ void write_box32(uint32_t box, int lane, const float 
   }
 }
 
+template <bool kEnt>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     lmhead_bwd_pair_kernel(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_wz,
                            const __grid_constant__ CUtensorMap tm_wn, const __grid_constant__ CUtensorMap tm_dh,
@@ -325,7 +327,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int v0 = un.vc * 256;
       const int row = own_row0 + r_in;
       const float coef = own_null ? 0.f : a.coef[row];
-      const float lseL = (coef != 0.f) ? a.lse[row] * kLog2e : 0.f;
+      float ecoef = 0.f, mu = 0.f;
+      if constexpr (kEnt) {
+        if (!own_null) {
+          ecoef = a.ecoef[row];
+          mu = a.mu[row];
+        }
+      }
+      const bool live = kEnt ? (coef != 0.f || ecoef != 0.f) : (coef != 0.f);
+      const float lseL = live ? a.lse[row] * kLog2e : 0.f;
       const int lx = a.tok_p[row] - v0;
       const int R = static_cast<int>(rank) * 128 + r_in;   // row of this token in GW
       // Z buffer -> g in GH (own tokens x 256 vocab) and GW (this / the peer CTA)
@@ -337,13 +347,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         float v[32];
         tmem_ld32(zaddr + c0, v);
         uint32_t w[16];
-        if (coef != 0.f) {
+        if (live) {
           const int lxc = lx - c0;
           const int nvalid = V - v0 - c0;
 #pragma unroll
           for (int j = 0; j < 32; j += 2) {
-            float g0 = coef * ex2_approx(fmaf(v[j], kLog2e, -lseL));
-            float g1 = coef * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+            float g0, g1;
+            if constexpr (kEnt) {   // p (coef + ecoef (z - mu)): the entropy-bonus term
+              g0 = fmaf(ecoef, v[j] - mu, coef) * ex2_approx(fmaf(v[j], kLog2e, -lseL));
+              g1 = fmaf(ecoef, v[j + 1] - mu, coef) * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+            } else {
+              g0 = coef * ex2_approx(fmaf(v[j], kLog2e, -lseL));
+              g1 = coef * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+            }
             if (j == lxc) g0 -= coef;
             if (j + 1 == lxc) g1 -= coef;
             if (j >= nvalid) g0 = 0.f;
@@ -413,14 +429,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 int lmhead_bwd_pair_max_clusters(int n_sm) {
   static int cached = -1;
   if (cached >= 0) return cached;
-  cudaError_t e = cudaFuncSetAttribute(lmhead_bwd_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  cudaError_t e =
+      cudaFuncSetAttribute(lmhead_bwd_pair_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return 0;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(n_sm, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = kSmemBytes;
   int n = 0;
-  e = cudaOccupancyMaxActiveClusters(&n, lmhead_bwd_pair_kernel, &cfg);
+  e = cudaOccupancyMaxActiveClusters(&n, lmhead_bwd_pair_kernel<false>, &cfg);
   if (e != cudaSuccess) {
     cudaGetLastError();
     n = n_sm / 2;
@@ -432,12 +449,19 @@ int lmhead_bwd_pair_max_clusters(int n_sm) {
 cudaError_t launch_lmhead_bwd_pair(const CUtensorMap& tm_h, const CUtensorMap& tm_w_z128, const CUtensorMap& tm_w_n,
                                    const CUtensorMap& tm_dh, const CUtensorMap& tm_dw, const BwdArgs& a, int n_sm,
                                    cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(lmhead_bwd_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  const bool ent = a.ecoef != nullptr;
+  cudaError_t e = ent ? cudaFuncSetAttribute(lmhead_bwd_pair_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSmemBytes)
+                      : cudaFuncSetAttribute(lmhead_bwd_pair_kernel<false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return e;
   int clusters = lmhead_bwd_pair_max_clusters(n_sm);
   if (clusters > n_sm / 2) clusters = n_sm / 2;
   if (clusters < 1) clusters = 1;
-  lmhead_bwd_pair_kernel<<<2 * clusters, kThreads, kSmemBytes, s>>>(tm_h, tm_w_z128, tm_w_n, tm_dh, tm_dw, a);
+  if (ent)
+    lmhead_bwd_pair_kernel<true><<<2 * clusters, kThreads, kSmemBytes, s>>>(tm_h, tm_w_z128, tm_w_n, tm_dh, tm_dw, a);
+  else
+    lmhead_bwd_pair_kernel<false><<<2 * clusters, kThreads, kSmemBytes, s>>>(tm_h, tm_w_z128, tm_w_n, tm_dh, tm_dw, a);
   return cudaGetLastError();
 }
 

@@ -32,6 +32,12 @@ struct Workspace {
   int32_t* tile_list;   // [Tcap/128]
   double* red;          // [n_tiles * kRedSlots] per-tile partial sums
   float* dh32;          // [Tcap, H] fp32 dhidden accumulator (loss call only)
+  // extended objective (loss call only)
+  float* lp_p;          // [Tcap] packed log-probs
+  float* ent_p;         // [Tcap] packed entropies
+  float* ecoef;         // [Tcap] m w entropy_coef / D
+  float* mu;            // [Tcap] sum_v p_v z_v = lse - entropy
+  uint8_t* gate_p;      // [Tcap] sequence-gate weight per packed row
 };
 constexpr int kRedSlots = 8;
 
@@ -59,7 +65,18 @@ struct BwdArgs {
   int V, H;
   int n_vchunks;
   int tile_group;            // token tiles per raster group
+  const float* ecoef;        // entropy-bonus coefficient per row, or nullptr
+  const float* mu;           // sum_v p_v z_v per row (with ecoef)
   unsigned* err;
+};
+
+// options of the extended objective as the row kernels see them
+struct LossEx {
+  float kl_coef;
+  float entropy_coef;
+  const float* ref_logp;     // [T] original order
+  const int32_t* seq;        // [T] original order, or nullptr
+  double gate_lo, gate_hi;
 };
 
 // api.cu: shared host helpers
@@ -83,7 +100,13 @@ cudaError_t launch_merge(bool loss_mode, int Tcap, int V, int n_split, double de
                          const Workspace& ws, float* logp_out, float* ent_out, float* tokloss_out, unsigned* err,
                          cudaStream_t s);
 cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* loss_out, void* stats_out,
-                            unsigned* err, cudaStream_t s);
+                            void* stats_ex_out, unsigned* err, cudaStream_t s);
+// extended objective: packed stats -> sequence gate -> loss rows
+cudaError_t launch_merge_stats_ex(int Tcap, int V, int n_split, const Workspace& ws, float* logp_out, float* ent_out,
+                                  unsigned* err, cudaStream_t s);
+cudaError_t launch_seq_gate(int T, int Tcap, const LossEx& ex, const Workspace& ws, unsigned* err, cudaStream_t s);
+cudaError_t launch_loss_rows_ex(int Tcap, double denom, float clip_lo, float clip_hi, const LossEx& ex,
+                                const Workspace& ws, float* tokloss_out, cudaStream_t s);
 cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s);
 
 // lmhead_fwd.cu

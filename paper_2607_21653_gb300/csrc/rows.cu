@@ -193,6 +193,7 @@ __global__ void __launch_bounds__(1024) compact_kernel(const uint8_t* __restrict
   if (threadIdx.x == 0) {
     counts[0] = total;
     counts[1] = 0;
+    counts[2] = 0;
   }
 }
 
@@ -258,7 +259,8 @@ __global__ void __launch_bounds__(128) merge_kernel(
     const float* __restrict__ b_p, const float* __restrict__ adv_p, const float4* __restrict__ part,
     const float* __restrict__ zx, float* __restrict__ lse_o, float* __restrict__ coef_o,
     int32_t* __restrict__ tile_flag, double* __restrict__ red, float* __restrict__ logp_out,
-    float* __restrict__ ent_out, float* __restrict__ tokloss_out, unsigned* err) {
+    float* __restrict__ ent_out, float* __restrict__ tokloss_out, float* __restrict__ lp_p,
+    float* __restrict__ ent_p, unsigned* err) {
   __shared__ double shd[4];
   __shared__ long long shl[4];
   const int n = counts[0];
@@ -307,6 +309,8 @@ __global__ void __launch_bounds__(128) merge_kernel(
     if (logp_out) logp_out[t] = logp;
     if (ent_out) ent_out[t] = ent;
     if (tokloss_out) tokloss_out[t] = tl;
+    if (lp_p) lp_p[k] = logp;
+    if (ent_p) ent_p[k] = ent;
   }
   if (!loss_mode) return;
   if (k < Tcap) coef_o[k] = coef;
@@ -326,6 +330,140 @@ __global__ void __launch_bounds__(128) merge_kernel(
     r[3] = m_alr;
     r[4] = static_cast<double>(c_lo);
     r[5] = static_cast<double>(c_hi);
+    r[6] = 0.0;
+    r[7] = 0.0;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Extended objective (Sec. 4.5: KL control, rejection rules).
+// ---------------------------------------------------------------------------
+
+// Sequence gate.  Thread i checks that the ids do not decrease at token i; warp
+// w owns packed rows [32 w, 32 w + 32) and handles every sequence that starts
+// there: it walks the sequence 32 packed rows at a time (packing keeps the
+// original order, so a sequence is a run of packed rows), sums logp - b in
+// fp64 with a fixed shuffle tree, and writes the gate weight of every row.
+// Reject when exp(mean) lies outside [lo, hi].
+__global__ void __launch_bounds__(256) seq_gate_kernel(int T, const int32_t* __restrict__ seq,
+                                                       const int32_t* __restrict__ counts,
+                                                       const int32_t* __restrict__ row_map,
+                                                       const float* __restrict__ lp_p, const float* __restrict__ b_p,
+                                                       double lo, double hi, uint8_t* __restrict__ gate_p,
+                                                       int32_t* __restrict__ n_rej, unsigned* err) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  if (i < T && i > 0 && seq[i] < seq[i - 1]) atomicOr(err, kDevErrUnsortedGroups);
+  const int n = counts[0];
+  const int base = i - lane;
+  if (base >= n) return;   // whole warp leaves together
+  const int k = base + lane;
+  const int sid = (k < n) ? seq[row_map[k]] : 0;
+  const bool start = (k < n) && (k == 0 || seq[row_map[k - 1]] != sid);
+  unsigned starts = __ballot_sync(0xffffffffu, start);
+  while (starts) {
+    const int s0 = base + __ffs(starts) - 1;
+    starts &= starts - 1;
+    const int sid0 = __shfl_sync(0xffffffffu, sid, s0 - base);
+    double acc = 0.0;
+    int len = 0;
+    for (int w0 = s0;; w0 += 32) {
+      const int kk = w0 + lane;
+      const bool in = kk < n && seq[row_map[kk]] == sid0;
+      const unsigned m = __ballot_sync(0xffffffffu, in);
+      const int run = (m == 0xffffffffu) ? 32 : __ffs(~m) - 1;   // leading rows of this sequence
+      double v = (lane < run) ? static_cast<double>(lp_p[kk]) - static_cast<double>(b_p[kk]) : 0.0;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+      acc += v;
+      len += run;
+      if (run < 32) break;
+    }
+    const double g = exp(acc / static_cast<double>(len));
+    const uint8_t keep = (g < lo || g > hi) ? 0 : 1;
+    for (int j = s0 + lane; j < s0 + len; j += 32) gate_p[j] = keep;
+    if (lane == 0 && !keep) atomicAdd(n_rej, 1);
+  }
+}
+
+// One block of 128 threads per packed tile: the per-token loss of the extended
+// objective and the two backward coefficients
+//   coef  = m w (c + kl_coef (e^r - 1)) / D      on (p - onehot)
+//   ecoef = m w entropy_coef / D                 on p (z - mu),  mu = lse - H
+__global__ void __launch_bounds__(128) loss_rows_ex_kernel(
+    int Tcap, double denom, float clip_lo, float clip_hi, LossEx ex, const int32_t* __restrict__ counts,
+    const int32_t* __restrict__ row_map, const float* __restrict__ b_p, const float* __restrict__ adv_p,
+    const float* __restrict__ lp_p, const float* __restrict__ ent_p, const float* __restrict__ lse,
+    const uint8_t* __restrict__ gate_p, float* __restrict__ coef_o, float* __restrict__ ecoef_o,
+    float* __restrict__ mu_o, int32_t* __restrict__ tile_flag, double* __restrict__ red,
+    float* __restrict__ tokloss_out) {
+  __shared__ double shd[4];
+  __shared__ long long shl[4];
+  const int n = counts[0];
+  const int n_tiles = (n + kTileM - 1) / kTileM;
+  if ((int)blockIdx.x >= n_tiles) return;
+  const int k = blockIdx.x * kTileM + threadIdx.x;
+  const bool act = k < n;
+  const double D = denom > 0.0 ? denom : static_cast<double>(n);
+  float coef = 0.f, ecoef = 0.f, mu = 0.f, tl = 0.f, ratio = 0.f, ent = 0.f, kl = 0.f;
+  int clip_lo_hit = 0, clip_hi_hit = 0, rejected = 0;
+  double alr = 0.0;
+  if (act) {
+    const float logp = lp_p[k], b = b_p[k], A = adv_p[k];
+    ent = ent_p[k];
+    ratio = expf(logp - b);
+    const float lo = 1.0f - clip_lo, hi = 1.0f + clip_hi;
+    const bool clipped = (A > 0.f && ratio > hi) || (A < 0.f && ratio < lo);
+    const float rc = fminf(fmaxf(ratio, lo), hi);
+    const float l_pg = clipped ? -(rc * A) : -(ratio * A);
+    const float c = clipped ? 0.f : ratio * A;
+    float c_kl = 0.f;
+    if (ex.kl_coef != 0.f) {
+      const float r = ex.ref_logp[row_map[k]] - logp;
+      const float em1 = expm1f(r);
+      kl = em1 - r;             // e^r - r - 1 without cancellation near r = 0
+      c_kl = ex.kl_coef * em1;
+    }
+    const bool keep = gate_p == nullptr || gate_p[k] != 0;
+    if (keep) {
+      tl = l_pg + ex.kl_coef * kl - ex.entropy_coef * ent;
+      coef = (D > 0.0) ? static_cast<float>(static_cast<double>(c + c_kl) / D) : 0.f;
+      ecoef = (D > 0.0) ? static_cast<float>(static_cast<double>(ex.entropy_coef) / D) : 0.f;
+      clip_lo_hit = (clipped && A < 0.f) ? 1 : 0;
+      clip_hi_hit = (clipped && A > 0.f) ? 1 : 0;
+    } else {
+      kl = 0.f;
+      rejected = 1;
+    }
+    mu = lse[k] - ent;
+    alr = fabs(static_cast<double>(logp) - static_cast<double>(b));
+    if (tokloss_out) tokloss_out[row_map[k]] = tl;
+  }
+  if (k < Tcap) {
+    coef_o[k] = coef;
+    ecoef_o[k] = ecoef;
+    mu_o[k] = mu;
+  }
+  const int any = __syncthreads_or(coef != 0.f || ecoef != 0.f);
+  double* rr = red + (int64_t)blockIdx.x * kRedSlots;
+  const double s_loss = block128_sum<double>(act ? (double)tl : 0.0, shd);
+  const double s_ratio = block128_sum<double>(act ? (double)ratio : 0.0, shd);
+  const double s_ent = block128_sum<double>(act ? (double)ent : 0.0, shd);
+  const double m_alr = block128_max(alr, shd);
+  const long long c_lo = block128_sum<long long>(clip_lo_hit, shl);
+  const long long c_hi = block128_sum<long long>(clip_hi_hit, shl);
+  const double s_kl = block128_sum<double>(act ? (double)kl : 0.0, shd);
+  const long long c_rej = block128_sum<long long>(rejected, shl);
+  if (threadIdx.x == 0) {
+    tile_flag[blockIdx.x] = any ? 1 : 0;
+    rr[0] = s_loss;
+    rr[1] = s_ratio;
+    rr[2] = s_ent;
+    rr[3] = m_alr;
+    rr[4] = static_cast<double>(c_lo);
+    rr[5] = static_cast<double>(c_hi);
+    rr[6] = s_kl;
+    rr[7] = static_cast<double>(c_rej);
   }
 }
 
@@ -333,6 +471,12 @@ struct StatsDev {
   double denom, loss, sum_ratio, sum_entropy, max_abs_log_ratio;
   long long n_active, n_clip_low, n_clip_high;
 };
+struct StatsExDev {
+  StatsDev base;
+  double sum_kl;
+  long long n_tokens_rejected, n_seq_rejected;
+};
+constexpr int kFinSlots = 8;
 
 // fixed-order reduction of the per-tile partials, the loss scalar, the stats
 // and the list of tiles whose rows have a nonzero gradient coefficient
@@ -340,45 +484,42 @@ __global__ void __launch_bounds__(1024) finalize_kernel(double denom, int32_t* _
                                                         const int32_t* __restrict__ tile_flag,
                                                         int32_t* __restrict__ tile_list,
                                                         const double* __restrict__ red, float* __restrict__ loss_out,
-                                                        StatsDev* __restrict__ stats, unsigned* err) {
-  __shared__ double sh[6][32];
+                                                        StatsDev* __restrict__ stats, StatsExDev* __restrict__ stats_ex,
+                                                        unsigned* err) {
+  __shared__ double sh[kFinSlots][32];
   const int n = counts[0];
   const int n_tiles = (n + kTileM - 1) / kTileM;
-  double a[6] = {0, 0, 0, 0, 0, 0};
+  double a[kFinSlots] = {0, 0, 0, 0, 0, 0, 0, 0};
   for (int b = threadIdx.x; b < n_tiles; b += blockDim.x) {
     const double* r = red + (int64_t)b * kRedSlots;
-    a[0] += r[0];
-    a[1] += r[1];
-    a[2] += r[2];
-    a[3] = fmax(a[3], r[3]);
-    a[4] += r[4];
-    a[5] += r[5];
+#pragma unroll
+    for (int q = 0; q < kFinSlots; ++q) a[q] = (q == 3) ? fmax(a[q], r[q]) : a[q] + r[q];
   }
   // fixed shuffle tree inside each warp, then warp 0 over the 32 warp results
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
 #pragma unroll
-    for (int q = 0; q < 6; ++q) {
+    for (int q = 0; q < kFinSlots; ++q) {
       const double y = __shfl_xor_sync(0xffffffffu, a[q], o);
       a[q] = (q == 3) ? fmax(a[q], y) : a[q] + y;
     }
   }
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   if (lane == 0)
-    for (int q = 0; q < 6; ++q) sh[q][w] = a[q];
+    for (int q = 0; q < kFinSlots; ++q) sh[q][w] = a[q];
   __syncthreads();
   if (w == 0) {
-    for (int q = 0; q < 6; ++q) a[q] = sh[q][lane];
+    for (int q = 0; q < kFinSlots; ++q) a[q] = sh[q][lane];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
 #pragma unroll
-      for (int q = 0; q < 6; ++q) {
+      for (int q = 0; q < kFinSlots; ++q) {
         const double y = __shfl_xor_sync(0xffffffffu, a[q], o);
         a[q] = (q == 3) ? fmax(a[q], y) : a[q] + y;
       }
     }
     if (lane == 0)
-      for (int q = 0; q < 6; ++q) sh[q][0] = a[q];
+      for (int q = 0; q < kFinSlots; ++q) sh[q][0] = a[q];
   }
   __syncthreads();
   const double D = denom > 0.0 ? denom : static_cast<double>(n);
@@ -395,6 +536,20 @@ __global__ void __launch_bounds__(1024) finalize_kernel(double denom, int32_t* _
       stats->n_active = n;
       stats->n_clip_low = static_cast<long long>(sh[4][0]);
       stats->n_clip_high = static_cast<long long>(sh[5][0]);
+    }
+    if (stats_ex) {
+      StatsDev& b = stats_ex->base;
+      b.denom = D;
+      b.loss = loss;
+      b.sum_ratio = sh[1][0];
+      b.sum_entropy = sh[2][0];
+      b.max_abs_log_ratio = sh[3][0];
+      b.n_active = n;
+      b.n_clip_low = static_cast<long long>(sh[4][0]);
+      b.n_clip_high = static_cast<long long>(sh[5][0]);
+      stats_ex->sum_kl = sh[6][0];
+      stats_ex->n_tokens_rejected = static_cast<long long>(sh[7][0]);
+      stats_ex->n_seq_rejected = counts[2];
     }
   }
   // compact the active tile list (order preserving)
@@ -488,15 +643,46 @@ cudaError_t launch_merge(bool loss_mode, int Tcap, int V, int n_split, double de
   const int blocks = Tcap / kTileM;
   merge_kernel<<<blocks, kTileM, 0, s>>>(loss_mode ? 1 : 0, Tcap, V, n_split, denom, clip_lo, clip_hi, ws.counts,
                                           ws.row_map, ws.tok_p, ws.b_p, ws.adv_p, ws.part, ws.zx, ws.lse, ws.coef,
-                                          ws.tile_flag, ws.red, logp_out, ent_out, tokloss_out, err);
+                                          ws.tile_flag, ws.red, logp_out, ent_out, tokloss_out, nullptr, nullptr,
+                                          err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_merge_stats_ex(int Tcap, int V, int n_split, const Workspace& ws, float* logp_out, float* ent_out,
+                                  unsigned* err, cudaStream_t s) {
+  const int blocks = Tcap / kTileM;
+  if (blocks == 0) return cudaSuccess;
+  merge_kernel<<<blocks, kTileM, 0, s>>>(0, Tcap, V, n_split, 0.0, 0.f, 0.f, ws.counts, ws.row_map, ws.tok_p, ws.b_p,
+                                          ws.adv_p, ws.part, ws.zx, ws.lse, ws.coef, ws.tile_flag, ws.red, logp_out,
+                                          ent_out, nullptr, ws.lp_p, ws.ent_p, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_seq_gate(int T, int Tcap, const LossEx& ex, const Workspace& ws, unsigned* err, cudaStream_t s) {
+  const int blocks = (Tcap + 255) / 256;
+  if (blocks == 0 || ex.seq == nullptr) return cudaSuccess;
+  seq_gate_kernel<<<blocks, 256, 0, s>>>(T, ex.seq, ws.counts, ws.row_map, ws.lp_p, ws.b_p, ex.gate_lo, ex.gate_hi,
+                                         ws.gate_p, ws.counts + 2, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_loss_rows_ex(int Tcap, double denom, float clip_lo, float clip_hi, const LossEx& ex,
+                                const Workspace& ws, float* tokloss_out, cudaStream_t s) {
+  const int blocks = Tcap / kTileM;
+  if (blocks == 0) return cudaSuccess;
+  loss_rows_ex_kernel<<<blocks, kTileM, 0, s>>>(Tcap, denom, clip_lo, clip_hi, ex, ws.counts, ws.row_map, ws.b_p,
+                                                 ws.adv_p, ws.lp_p, ws.ent_p, ws.lse,
+                                                 ex.seq ? ws.gate_p : nullptr, ws.coef, ws.ecoef, ws.mu,
+                                                 ws.tile_flag, ws.red, tokloss_out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* loss_out, void* stats_out,
-                            unsigned* err, cudaStream_t s) {
+                            void* stats_ex_out, unsigned* err, cudaStream_t s) {
   (void)Tcap;
   finalize_kernel<<<1, 1024, 0, s>>>(denom, ws.counts, ws.tile_flag, ws.tile_list, ws.red, loss_out,
-                                     reinterpret_cast<StatsDev*>(stats_out), err);
+                                     reinterpret_cast<StatsDev*>(stats_out),
+                                     reinterpret_cast<StatsExDev*>(stats_ex_out), err);
   return cudaGetLastError();
 }
 

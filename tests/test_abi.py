@@ -73,3 +73,17 @@ def test_workspace_sizes_grow_with_problem(lib):
     assert molt.policy_loss_workspace_bytes(1000, 100, 4096) == 0   # unsupported H
     # dhidden fp32 accumulator + packed bf16 copy of the hidden rows dominate
     assert b >= 1024 * 256 * 6
+
+
+def test_rejects_bad_loss_options(lib):
+    opts = molt.LossOptions(0.1, 0.0, None, None, 0.0, 0.0)      # KL without ref_logp
+    args = [FAKE] * 6 + [16, 64, 32, 0.2, 0.2, 0.0, ctypes.byref(opts)] + [FAKE, FAKE, FAKE, 0, None, None, None,
+                                                                          None, None, 0, None]
+    assert molt.STATUS[lib.molt_policy_loss_fwd_bwd_ex(*args)] == "MOLT_ERR_INVALID_ARG"
+    assert "ref_logp" in lib.molt_last_error().decode()
+    opts = molt.LossOptions(0.0, 0.0, None, FAKE, 2.0, 1.0)      # empty gate band
+    args[12] = ctypes.byref(opts)
+    assert molt.STATUS[lib.molt_policy_loss_fwd_bwd_ex(*args)] == "MOLT_ERR_INVALID_ARG"
+    opts = molt.LossOptions(-1.0, 0.0, FAKE, None, 0.0, 0.0)     # negative KL weight
+    args[12] = ctypes.byref(opts)
+    assert molt.STATUS[lib.molt_policy_loss_fwd_bwd_ex(*args)] == "MOLT_ERR_INVALID_ARG"
