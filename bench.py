@@ -10,6 +10,13 @@ in spans of 8-256, clip eps 0.2 / 0.28.  Inputs are synthetic and seeded
 1.24 GB, larger than L2, so no extra flush runs between steps.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--estimator grpo|group_mean|dr_grpo|rloo|reinforce_pp]
+                  [--objective ppo|kl_entropy_gate]
+
+--estimator picks the advantage estimator (Sec. 4.5 list); --objective
+kl_entropy_gate adds a KL-to-reference term, an entropy bonus and the
+sequence-level importance gate (one sequence per rollout) to the loss.  The
+defaults are the headline configuration (GRPO, clipped surrogate).
 
 With torchrun (N > 1) every rank processes its own batch (different seed)
 with no collective on the data path ("scaling": "weak"); rank 0 prints.
@@ -34,6 +41,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "policy-loss fwd+bwd tokens/s on 1 GB300; % of dense bf16 tensor peak"
 KERNELS_PER_STEP = 9   # advantages, broadcast, compact, gather, forward, merge, finalize, backward, cast
+KERNELS_PER_STEP_EX = 11   # + sequence gate and loss rows (merge writes the packed row statistics)
 
 
 def load_peaks():
@@ -269,10 +277,28 @@ def run_ours(args):
     adv_tok = torch.empty(T, dtype=torch.float32, device=dev)
     dW = torch.empty(V, H, dtype=torch.float32, device=dev)
     n_active = int(w.mask.sum())
+    extended = args.objective == "kl_entropy_gate"
+    ex_opts = {}
+    if extended:
+        # reference-policy log-probs: the current ones plus an independent lag;
+        # one gated sequence per rollout; a band wide enough that the gate
+        # rejects (and so skips) no work at this behaviour lag
+        rnoise = np.random.default_rng(w.seed + 29).normal(0.0, 0.1, T).astype(np.float32)
+        ex_opts = dict(kl_coef=0.01, ref_logp=(lp + torch.from_numpy(rnoise).to(dev)).contiguous(),
+                       entropy_coef=1e-3, seq_of_token=rot, gate_lo=0.5, gate_hi=2.0)
 
-    def step(tok=tokens, msk=mask, hid=hidden, bb=b, rw=rewards, gi=gids, ro=rot):
-        molt.group_advantages(rw, gi, out=adv_resp)
+    def step(tok=tokens, msk=mask, hid=hidden, bb=b, rw=rewards, gi=gids, ro=rot, rf=None):
+        if args.estimator == "grpo":
+            molt.group_advantages(rw, gi, out=adv_resp)
+        else:
+            molt.advantages(rw, None if args.estimator == "reinforce_pp" else gi, estimator=args.estimator,
+                            out=adv_resp)
         molt.broadcast_advantages(adv_resp, ro, out=adv_tok)
+        if extended:
+            return molt.policy_loss_fwd_bwd_ex(hid, weight, tok, bb, adv_tok, msk, w.eps_lo, w.eps_hi, dW=dW,
+                                               want_token_outputs=False,
+                                               **dict(ex_opts, seq_of_token=ro,
+                                                      ref_logp=ex_opts["ref_logp"] if rf is None else rf))
         return molt.policy_loss_fwd_bwd(hid, weight, tok, bb, adv_tok, msk, w.eps_lo, w.eps_hi, dW=dW,
                                         want_token_outputs=False)
 
@@ -308,6 +334,7 @@ def run_ours(args):
     timer.close()
     assert molt.device_status() == 0
     loss_val = float(out["loss"].item())
+    step_stats = molt.stats_dict(out["stats"])
     ms = max_over_ranks(ms, world, dev)
 
     # ---- end to end through the public API with host buffers
@@ -321,29 +348,39 @@ def run_ours(args):
         d_tok, d_msk, d_b = torch.empty_like(tokens), torch.empty_like(mask), torch.empty_like(b)
         d_rw, d_gi, d_ro = torch.empty_like(rewards), torch.empty_like(gids), torch.empty_like(rot)
         h_loss = torch.empty(1, dtype=torch.float32).pin_memory()
-        h2d = sum(x.numel() * x.element_size() for x in (h_hid, h_tok, h_msk, h_b, h_rw, h_gi, h_ro))
+        copies = [(d_hid, h_hid), (d_tok, h_tok), (d_msk, h_msk), (d_b, h_b), (d_rw, h_rw), (d_gi, h_gi),
+                  (d_ro, h_ro)]
+        d_rf = None
+        if extended:
+            h_rf = pin(ex_opts["ref_logp"].cpu().numpy())
+            d_rf = torch.empty_like(ex_opts["ref_logp"])
+            copies.append((d_rf, h_rf))
+        h2d = sum(src.numel() * src.element_size() for _, src in copies)
         e_steps = max(1, args.steps // 2)
+        for dst, src in copies:
+            dst.copy_(src)
         for _ in range(2):
-            o = step(d_tok, d_msk, d_hid.view(torch.bfloat16), d_b, d_rw, d_gi, d_ro)
+            o = step(d_tok, d_msk, d_hid.view(torch.bfloat16), d_b, d_rw, d_gi, d_ro, d_rf)
         torch.cuda.synchronize()
         barrier()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
         for _ in range(e_steps):
-            for dst, src in ((d_hid, h_hid), (d_tok, h_tok), (d_msk, h_msk), (d_b, h_b), (d_rw, h_rw),
-                             (d_gi, h_gi), (d_ro, h_ro)):
+            for dst, src in copies:
                 dst.copy_(src, non_blocking=True)
-            o = step(d_tok, d_msk, d_hid.view(torch.bfloat16), d_b, d_rw, d_gi, d_ro)
+            o = step(d_tok, d_msk, d_hid.view(torch.bfloat16), d_b, d_rw, d_gi, d_ro, d_rf)
             h_loss.copy_(o["loss"], non_blocking=True)
         e1.record()
         torch.cuda.synchronize()
+        assert molt.device_status() == 0
         ems = e0.elapsed_time(e1)
         ems = max_over_ranks(ems, world, dev)
         e2e = {"value": job_throughput(T, world, e_steps, ems), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": 4, "steps": e_steps,
                "note": "hidden, tokens, mask, behaviour log-probs, rewards, group ids and the token->rollout map "
-                       "copied from pinned host memory every step; W stays resident; loss read back"}
+                       + ("(and reference log-probs) " if extended else "")
+                       + "copied from pinned host memory every step; W stays resident; loss read back"}
 
     if rank != 0:
         if world > 1:
@@ -359,11 +396,12 @@ def run_ours(args):
     achieved_bwd = 4.0 * tp * H * V / bwd_s / 1e12
     step_s = ms / 1e3 / args.steps
     step_frac = 6.0 * tp * H * V / step_s / 1e12 / peak
-    bwd_kernel = "lmhead_bwd_pair_kernel" if H % 256 == 0 else "lmhead_bwd_kernel"
+    bwd_kernel = "lmhead_bwd_quad_kernel" if H % 256 == 0 else "lmhead_bwd_kernel"
     roofline = {
         "kernel": bwd_kernel, "bound": "tensor", "achieved": achieved_bwd, "peak": peak, "unit": "TFLOP/s",
         "frac": achieved_bwd / peak, "traffic": recorded_traffic(bwd_kernel),
-        "limiter": "per-SM reduce-add egress of the fp32 partial products (~25 B/clock/SM measured)",
+        "limiter": "tensor issue: N=128 pair MMAs take ~1.6x their ideal cycles; operand-stage round trips "
+                   "(~2.5K clocks) with a 64 KB ring",
         "peak_source": f"{peaks['source']} bf16 sustained (kernel timed inside a long step)",
         "algorithmic_flops_per_launch": 4.0 * tp * H * V,
         "executed_tflops": 6.0 * tp * H * V / bwd_s / 1e12,
@@ -396,12 +434,14 @@ def run_ours(args):
                    "l2": "inputs larger than L2 (W 1.24 GB); no flush",
                    "tensor_peak_frac_6THV": step_frac,
                    "tensor_peak_frac_6THV_of_burst": 6.0 * tp * H * V / step_s / 1e12 / peaks["bf16"],
-                   "loss": loss_val},
+                   "loss": loss_val, "estimator": args.estimator, "objective": args.objective,
+                   **({"kl_coef": 0.01, "entropy_coef": 1e-3, "gate": [0.5, 2.0],
+                       "seq_rejected": step_stats.get("n_seq_rejected")} if extended else {})},
         "roofline": roofline,
         "cpu_baseline": cpu,
         "clocks": clk,
         "e2e": e2e,
-        "gpu_launches": KERNELS_PER_STEP * args.steps,
+        "gpu_launches": (KERNELS_PER_STEP_EX if extended else KERNELS_PER_STEP) * args.steps,
     }
     print(json.dumps(line), flush=True)
     if world > 1:
@@ -420,6 +460,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--ref-rows", type=int, default=32)
+    ap.add_argument("--estimator", default="grpo", choices=("grpo", "group_mean", "dr_grpo", "rloo", "reinforce_pp"))
+    ap.add_argument("--objective", default="ppo", choices=("ppo", "kl_entropy_gate"))
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

@@ -93,15 +93,16 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 
 // 2-D row-major tensor map: `rows` x `cols` elements, box `box_cols` x `box_rows`
 molt_status make_tmap(CUtensorMap* m, CUtensorMapDataType dt, int elem_bytes, const void* base, uint64_t rows,
-                      uint64_t cols, uint32_t box_cols, uint32_t box_rows) {
+                      uint64_t cols, uint32_t box_cols, uint32_t box_rows,
+                      CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   auto fn = encode_fn();
   if (!fn) return fail(MOLT_ERR_CUDA, "cuTensorMapEncodeTiled entry point unavailable");
   cuuint64_t dims[2] = {cols, rows};
   cuuint64_t strides[1] = {cols * static_cast<uint64_t>(elem_bytes)};
   cuuint32_t box[2] = {box_cols, box_rows};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                  CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  CUresult r = fn(m, dt, 2, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(MOLT_ERR_CUDA, "cuTensorMapEncodeTiled failed (" + std::to_string((int)r) + ")");
   return MOLT_OK;
 }
@@ -324,6 +325,11 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
   MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, pair_bwd ? 128 : kBwdBV));
   MOLT_TRY(make_tmap(&tm_wn, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, 64));
+  // 64-byte-swizzled K = 32 boxes of h and W for the logit recompute on CTA pairs
+  CUtensorMap tm_hz, tm_wz32;
+  MOLT_TRY(make_tmap(&tm_hz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, 32, kTileM,
+                     CU_TENSOR_MAP_SWIZZLE_64B));
+  MOLT_TRY(make_tmap(&tm_wz32, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, 32, 128, CU_TENSOR_MAP_SWIZZLE_64B));
   MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
   MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
   MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
@@ -357,7 +363,9 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   ba.V = static_cast<int>(V);
   ba.H = static_cast<int>(H);
   ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
-  ba.tile_group = pair_bwd ? 8 : 16;
+  ba.tile_group = pair_bwd ? 4 : 16;
+  ba.dh32 = w.dh32;
+  ba.dW = dW_out;   // token tiles: 4 quads (2048 rows) or 16 tiles per raster group
   if (opts && ex.entropy_coef != 0.f) {
     ba.ecoef = w.ecoef;
     ba.mu = w.mu;
@@ -365,7 +373,8 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   ba.err = di->status;
   ev_start(3, stream);
   if (pair_bwd)
-    MOLT_CUDA(launch_lmhead_bwd_pair(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+    MOLT_CUDA(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
+              "lmhead backward");
   else
     MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
   ev_stop(3, stream);

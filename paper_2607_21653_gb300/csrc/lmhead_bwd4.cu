@@ -1,0 +1,576 @@
+// Backward pass of the fused LM-head + policy loss on clusters of four CTAs
+// (two tcgen05 CTA pairs), used when H is a multiple of 256.
+//
+//   g_tv = coef_t (softmax(z_t)_v - [v == x_t]),  coef_t = m_t c_t / D   (Eq. 2)
+//          (+ ecoef_t softmax(z_t)_v (z_tv - mu_t) with an entropy bonus)
+//   dH_t = sum_v g_tv W_v          dW_v = sum_t g_tv h_t
+//
+// Why clusters of four.  The products of a unit are partial sums over its
+// slice of the reduction dimension (vocab for dH, tokens for dW), so every unit
+// drains H-wide fp32 rows into global memory with reduce-adds.  Those drains,
+// together with the operand loads, go through each SM's request path to L2,
+// which moves about 32 B per clock, and that path, not the tensor cores, is what
+// bounds this kernel.  A unit of Tu tokens x Vu vocab drains 4 H (Tu + Vu) bytes
+// for 6 Tu Vu H flops, so larger units drain less per flop.  The on-chip state
+// that has to grow with the unit is g, which is small (bf16, no H dimension):
+// here a unit is 512 tokens x 512 vocab on four CTAs, twice as deep in both
+// reductions as a 256 x 256 unit on one CTA pair, which halves the drain bytes
+// per flop.  The price is moving g between the CTAs through distributed shared
+// memory (96 KB per CTA per unit, against 4 MB of drains).
+//
+// Layout of a unit.  CTA k (cluster rank k = 0..3) owns token tile k of the
+// unit's four 128-row tiles and vocab quarter k (columns v0 + 128 k ...).  Pair
+// p = k / 2 (CTAs 2p, 2p+1) computes, on the tensor cores of both its SMs:
+//   Z      z = h W^T for its two token tiles x all 512 vocab, as two pair MMAs
+//          of M = 256 tokens, N = 256 vocab (Z_a: vocab 0..255, Z_b: 256..511),
+//          K = H.  Each CTA's TMEM receives its 128 tokens x 256 vocab.
+//   g      each CTA turns z into g (bf16): into TMEM (its 128 tokens x 512 vocab,
+//          256 columns, the A operand of dH) and into the GW buffers of all four
+//          CTAs: the GW of CTA q holds g of all 512 tokens x vocab quarter q
+//          (MN-major A operand of dW), filled by every CTA for its own tokens.
+//   dH     per 128 columns of H: pair MMA M = 256 tokens, N = 128, K = 512 vocab;
+//          A = g from TMEM, B = W rows (MN-major), CTA r staging columns
+//          64 r .. 64 r + 63.
+//   dW     per 128 columns of H: pair MMA M = 256 vocab (the pair's two
+//          quarters), N = 128, K = 512 tokens; A = GW, B = h rows of all four
+//          tiles (MN-major).
+// Partial products drain through swizzled 32 x 32 fp32 boxes with TMA
+// reduce-add into the fp32 dhidden accumulator and dW.
+//
+// TMEM (512 columns per CTA): [0, 256) g; [256, 384) and [384, 512) the job
+// accumulators.  Z_a accumulates over [0, 256) and Z_b over [128, 384); each is
+// converted to g in place (column c of z -> column c / 2 of g), so Z_a of the
+// next unit is computed while the current dW products run, and Z_b once the
+// accumulators are idle.  The epilogue copies each accumulator to registers and
+// hands it back before draining, so one free accumulator keeps the MMAs going.
+//
+// Operands stream through a ring of four 16 KB stages.  Every stage is a round
+// trip (the MMA frees it, the producer refills it from L2), and the ring's
+// bytes in flight over that latency set the rate at which operands arrive, so
+// the ring is cut fine: a logit stage holds K = 32 of h and W in the 64-byte
+// swizzle, a dH stage 128 vocab rows of W, a dW stage one token tile of h.
+//
+// Roles per CTA (192 threads): warp 0 TMA producer (each CTA loads its half of
+// every operand; bytes complete on the pair leader's barrier), warp 1 MMA issuer
+// (pair leaders only) and TMEM owner, warps 2-5 epilogue.
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "molt_internal.cuh"
+#include "ptx.cuh"
+
+namespace molt {
+namespace {
+
+constexpr int kStages = 4;
+constexpr int kStageBytes = 16 * 1024;
+constexpr int kSub = kTileM * kBK * 2;            // [128 rows x 64] bf16 sub-tile, 16 KB
+constexpr int kZK = 32;                           // K per logit stage (64-byte swizzle rows)
+constexpr int kOffGW = kStages * kStageBytes;     // 64 KB (1024-aligned)
+constexpr int kGWBlock = 4 * kSub;                // [512 token rows x 64 vocab] bf16, 64 KB
+constexpr int kOffBox = kOffGW + 2 * kGWBlock;    // 192 KB
+constexpr int kBoxBytes = 32 * 32 * 4;
+constexpr int kBoxesPerWarp = 2;
+constexpr int kThreads = 192;
+constexpr int kSmemBytes = 1024 + kOffBox + 4 * kBoxesPerWarp * kBoxBytes;
+constexpr uint32_t kIdescZ = idesc_bf16_f32(256, 256, false, false);
+constexpr uint32_t kIdescH = idesc_bf16_f32(256, 128, false, true);   // A from TMEM
+constexpr uint32_t kIdescW = idesc_bf16_f32(256, 128, true, true);
+constexpr uint32_t kGCol = 0;       // g: 128 tokens x 512 vocab as bf16 pairs
+constexpr uint32_t kZaCol = 0;      // Z of vocab 0..255
+constexpr uint32_t kZbCol = 128;    // Z of vocab 256..511
+constexpr uint32_t kAccCol = 256;   // two 128-column job accumulators
+constexpr uint32_t kStageTx = 2u * kStageBytes;   // bytes both CTAs of a pair load per stage
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct QuadUnit {
+  int tq;   // token-tile quad
+  int vp;   // 512-column vocab block
+};
+
+// raster: tile quads in groups of `group`; inside a group consecutive units walk
+// the group's quads for one vocab block, then move to the next block
+__device__ __forceinline__ QuadUnit quad_unit_of(int u, int n_tq, int n_vp, int group) {
+  const int per_group = group * n_vp;
+  const int g = u / per_group;
+  const int r = u - g * per_group;
+  const int g_q = min(group, n_tq - g * group);
+  const int vp = r / g_q;
+  return {g * group + (r - vp * g_q), vp};
+}
+
+__device__ __forceinline__ void write_box32(uint32_t box, int lane, const float (&v)[32]) {
+  const uint32_t rowp = box + lane * 128;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t pos = static_cast<uint32_t>(i ^ (lane & 7));
+    st_shared_v4(rowp + pos * 16, __float_as_uint(v[4 * i]), __float_as_uint(v[4 * i + 1]),
+                 __float_as_uint(v[4 * i + 2]), __float_as_uint(v[4 * i + 3]));
+  }
+}
+
+template <bool kEnt>
+__global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
+    lmhead_bwd_quad_kernel(const __grid_constant__ CUtensorMap tm_hz, const __grid_constant__ CUtensorMap tm_wz,
+                           const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_wn,
+                           const __grid_constant__ CUtensorMap tm_dh, const __grid_constant__ CUtensorMap tm_dw,
+                           const BwdArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ __align__(8) uint64_t full_bar[kStages];   // pair leader: both CTAs' bytes land here
+  __shared__ __align__(8) uint64_t empty_bar[kStages];  // both CTAs of the pair
+  __shared__ __align__(8) uint64_t accf_bar[2];         // both CTAs of the pair: accumulator full
+  __shared__ __align__(8) uint64_t acce_bar[2];         // pair leader: 256 epilogue arrivals
+  __shared__ __align__(8) uint64_t zfa_bar;             // every CTA: Z_a done in both pairs (2 commits)
+  __shared__ __align__(8) uint64_t zfb_bar;             // every CTA: Z_b done in both pairs (2 commits)
+  __shared__ __align__(8) uint64_t ta_bar;              // pair leader: Z_a read, g_a in TMEM (256)
+  __shared__ __align__(8) uint64_t tb_bar;              // pair leader: Z_b read, g_b in TMEM (256)
+  __shared__ __align__(8) uint64_t gw_bar;              // pair leader: both GW buffers of the pair full (512)
+  __shared__ __align__(8) uint64_t dhd_bar;             // pair leader: this unit's dH products done
+  __shared__ __align__(8) uint64_t done_bar;
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ int abort_sh;
+
+  const uint32_t smem0 = (smem_u32(smem_raw) + 1023u) & ~1023u;
+  const uint32_t gw_base = smem0 + kOffGW;
+  const uint32_t box_base = smem0 + kOffBox;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();   // token tile and vocab quarter of this CTA
+  const uint32_t prank = rank & 1u;          // rank inside the pair
+  const uint32_t lead = rank & ~1u;          // the pair leader's rank
+  const bool leader = prank == 0;
+  const uint16_t pair_mask = static_cast<uint16_t>(3u << lead);
+  volatile int* abort_flag = &abort_sh;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_u32(&full_bar[s]), 1);
+      mbar_init(smem_u32(&empty_bar[s]), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(smem_u32(&accf_bar[b]), 1);
+      mbar_init(smem_u32(&acce_bar[b]), 256);
+    }
+    mbar_init(smem_u32(&zfa_bar), 2);
+    mbar_init(smem_u32(&zfb_bar), 2);
+    mbar_init(smem_u32(&ta_bar), 256);
+    mbar_init(smem_u32(&tb_bar), 256);
+    mbar_init(smem_u32(&gw_bar), 512);
+    mbar_init(smem_u32(&dhd_bar), 1);
+    mbar_init(smem_u32(&done_bar), 1);
+    abort_sh = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(&tmem_base_sh), 512);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();   // every CTA's barriers exist before any remote arrival
+  tc_fence_after();
+  const uint32_t tmem_base = tmem_base_sh;
+
+  const int n_tiles = a.counts[1];
+  const int n_tq = (n_tiles + 3) / 4;
+  const int n_vp = (a.V + 511) / 512;
+  const int n_units = n_tq * n_vp;
+  const int H = a.H, V = a.V;
+  const int nZ = H / kZK;        // logit stages per vocab half (4 per dW job)
+  const int nJ = H / 128;        // dH jobs = dW jobs per unit
+  const int quad = blockIdx.x >> 2, n_quads = gridDim.x >> 2;
+
+  // token tile k of unit tq (a missing tile reads tile 0's rows; its g is 0)
+  auto tile_of = [&](int tq, int k) -> int {
+    const int i = 4 * tq + k;
+    return a.tile_list[i < n_tiles ? i : 4 * tq];
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      prefetch_tmap(&tm_hz);
+      prefetch_tmap(&tm_wz);
+      prefetch_tmap(&tm_h);
+      prefetch_tmap(&tm_wn);
+      uint32_t full_leader[kStages];
+      for (int s = 0; s < kStages; ++s) full_leader[s] = mapa_shared(smem_u32(&full_bar[s]), lead);
+      uint32_t it = 0;
+      bool ok = true;
+      auto next_stage = [&](uint32_t& sa, uint32_t& fb) -> bool {
+        const uint32_t st = it % kStages, ph = (it / kStages) & 1u;
+        if (!mbar_wait(smem_u32(&empty_bar[st]), ph ^ 1u, abort_flag, a.err)) return false;
+        sa = smem0 + st * kStageBytes;
+        fb = full_leader[st];
+        if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[st]), kStageTx);
+        ++it;
+        return true;
+      };
+      // one logit stage: K = 32 of the own token rows and of this CTA's 128 of
+      // the half's 256 vocab rows
+      auto load_z = [&](int kb, int own_row0, int vrow0) -> bool {
+        uint32_t sa, fb;
+        if (!next_stage(sa, fb)) return false;
+        tma_load_2d_pair(sa, &tm_hz, fb, kb * kZK, own_row0);
+        tma_load_2d_pair(sa + kStageBytes / 2, &tm_wz, fb, kb * kZK, vrow0 + static_cast<int>(prank) * 128);
+        return true;
+      };
+      int u = quad;
+      if (u < n_units) {
+        const QuadUnit un = quad_unit_of(u, n_tq, n_vp, a.tile_group);
+        const int own_row0 = tile_of(un.tq, static_cast<int>(rank)) * kTileM;
+        for (int kb = 0; kb < nZ && ok; ++kb) ok = load_z(kb, own_row0, un.vp * 512);
+      }
+      for (; u < n_units && ok; u += n_quads) {
+        const QuadUnit un = quad_unit_of(u, n_tq, n_vp, a.tile_group);
+        const int v0 = un.vp * 512;
+        const int own_row0 = tile_of(un.tq, static_cast<int>(rank)) * kTileM;
+        int t4[4];
+        for (int k = 0; k < 4; ++k) t4[k] = tile_of(un.tq, k) * kTileM;
+        const int un_next = u + n_quads;
+        int n_row0 = 0, n_v0 = 0;
+        if (un_next < n_units) {
+          const QuadUnit nu = quad_unit_of(un_next, n_tq, n_vp, a.tile_group);
+          n_row0 = tile_of(nu.tq, static_cast<int>(rank)) * kTileM;
+          n_v0 = nu.vp * 512;
+        }
+        // Z_b of this unit
+        for (int kb = 0; kb < nZ && ok; ++kb) ok = load_z(kb, own_row0, v0 + 256);
+        // dH jobs: W rows of the unit's 512 vocab, 128 per stage, this CTA's 64
+        // of 128 columns
+        for (int i = 0; i < nJ && ok; ++i) {
+          const int x = i * 128 + static_cast<int>(prank) * 64;
+          for (int st = 0; st < 4 && ok; ++st) {
+            uint32_t sa, fb;
+            if (!(ok = next_stage(sa, fb))) break;
+            tma_load_2d_pair(sa, &tm_wn, fb, x, v0 + st * 128);
+            tma_load_2d_pair(sa + 8192, &tm_wn, fb, x, v0 + st * 128 + 64);
+          }
+        }
+        // dW jobs: h rows of the four tiles, one per stage, this CTA's 64 of 128
+        // columns; the next unit's Z_a stages in between
+        for (int j = 0; j < nJ && ok; ++j) {
+          const int x = j * 128 + static_cast<int>(prank) * 64;
+          for (int st = 0; st < 4 && ok; ++st) {
+            uint32_t sa, fb;
+            if (!(ok = next_stage(sa, fb))) break;
+            tma_load_2d_pair(sa, &tm_h, fb, x, t4[st]);
+          }
+          if (un_next < n_units)
+            for (int kb = 4 * j; kb < 4 * j + 4 && ok; ++kb) ok = load_z(kb, n_row0, n_v0);
+        }
+      }
+      if (leader) {
+        // every copy of both CTAs completes on these barriers: wait for the
+        // last issued stages before the pair may exit
+        const uint32_t first = it > (uint32_t)kStages ? it - kStages : 0u;
+        for (uint32_t j = first; j < it; ++j)
+          mbar_wait_drain(smem_u32(&full_bar[j % kStages]), (j / kStages) & 1u, a.err);
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      uint32_t it = 0, jj = 0, unit_it = 0;
+      bool ok = true;
+      auto wait_stage = [&](uint32_t& sa) -> bool {
+        const uint32_t st = it % kStages, ph = (it / kStages) & 1u;
+        // the copies' complete_tx makes both CTAs' bytes visible to the MMAs
+        // issued after the phase flips; a CTA-scope wait is enough
+        if (!mbar_wait(smem_u32(&full_bar[st]), ph, abort_flag, a.err)) return false;
+        tc_fence_after();
+        sa = smem0 + st * kStageBytes;
+        return true;
+      };
+      auto release_stage = [&]() {
+        umma_commit_pair_mc(smem_u32(&empty_bar[it % kStages]), pair_mask);
+        ++it;
+      };
+      // one logit stage into the TMEM columns at zcol; the last one signals
+      // every CTA of the cluster through `bar`
+      auto z_block = [&](int kb, uint32_t zcol, uint32_t bar) -> bool {
+        uint32_t sa;
+        if (!wait_stage(sa)) return false;
+        const uint64_t ad = sdesc_sw64(sa);
+        const uint64_t bd = sdesc_sw64(sa + kStageBytes / 2);
+#pragma unroll
+        for (int k = 0; k < kZK / 16; ++k)
+          umma_bf16_pair(tmem_base + zcol, ad + 2u * k, bd + 2u * k, kIdescZ, (kb | k) != 0 ? 1u : 0u);
+        release_stage();
+        if (kb == nZ - 1) umma_commit_pair_mc(bar, 0xF);
+        return true;
+      };
+      // wait until accumulator `buf` may be written by job index j
+      auto acc_free = [&](uint32_t j) -> bool {
+        const uint32_t buf = j & 1u, aph = (j >> 1) & 1u;
+        if (!mbar_wait(smem_u32(&acce_bar[buf]), aph ^ 1u, abort_flag, a.err)) return false;
+        tc_fence_after();
+        return true;
+      };
+      int u = quad;
+      if (u < n_units)
+        for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
+      for (; u < n_units && ok; u += n_quads) {
+        const bool has_next = u + n_quads < n_units;
+        // Z_b over [128, 384): Z_a read by both CTAs and both accumulators idle
+        if (!(ok = mbar_wait_cluster(smem_u32(&ta_bar), unit_it & 1u, abort_flag, a.err))) break;
+        if (!(ok = acc_free(jj) && acc_free(jj + 1))) break;
+        for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb, kZbCol, smem_u32(&zfb_bar));
+        if (!ok) break;
+        // dH: A = g from TMEM (K = 512 vocab), B = W rows (MN-major)
+        if (!(ok = mbar_wait_cluster(smem_u32(&tb_bar), unit_it & 1u, abort_flag, a.err))) break;
+        tc_fence_after();
+        for (int i = 0; i < nJ && ok; ++i) {
+          if (!(ok = acc_free(jj))) break;
+          const uint32_t buf = jj & 1u;
+          const uint32_t d = tmem_base + kAccCol + buf * 128;
+          for (int st = 0; st < 4 && ok; ++st) {   // 128 vocab rows per stage
+            uint32_t sa;
+            if (!(ok = wait_stage(sa))) break;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const int vb = k >> 2, kk = k & 3;
+              const uint64_t bd = sdesc_sw128(sa + vb * 8192 + kk * 2048, 8192, 1024);
+              umma_bf16_pair_ta(d, tmem_base + kGCol + 8u * static_cast<uint32_t>(st * 8 + k), bd, kIdescH,
+                                (st | k) != 0 ? 1u : 0u);
+            }
+            release_stage();
+          }
+          umma_commit_pair_mc(smem_u32(&accf_bar[buf]), pair_mask);
+          ++jj;
+        }
+        if (!ok) break;
+        umma_commit_pair_mc(smem_u32(&dhd_bar), static_cast<uint16_t>(1u << rank));
+        // dW: A = g^T of the pair's two vocab quarters over 512 tokens (GW),
+        // B = h rows; the next unit's Z_a K-blocks in between
+        if (!(ok = mbar_wait_cluster(smem_u32(&gw_bar), unit_it & 1u, abort_flag, a.err))) break;
+        tc_fence_after();
+        for (int j = 0; j < nJ && ok; ++j) {
+          if (!(ok = acc_free(jj))) break;
+          const uint32_t buf = jj & 1u;
+          const uint32_t d = tmem_base + kAccCol + buf * 128;
+          for (int st = 0; st < 4 && ok; ++st) {   // one token tile per stage
+            uint32_t sa;
+            if (!(ok = wait_stage(sa))) break;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const uint64_t ad = sdesc_sw128(gw_base + (st * 8 + k) * 2048, kGWBlock, 1024);
+              const uint64_t bd = sdesc_sw128(sa + k * 2048, 16384, 1024);
+              umma_bf16_pair(d, ad, bd, kIdescW, (st | k) != 0 ? 1u : 0u);
+            }
+            release_stage();
+          }
+          umma_commit_pair_mc(smem_u32(&accf_bar[buf]), pair_mask);
+          ++jj;
+          if (has_next && ok) {
+            if (j == 0) {   // the dH products have read g: Z_a may overwrite it
+              if (!(ok = mbar_wait(smem_u32(&dhd_bar), unit_it & 1u, abort_flag, a.err))) break;
+              tc_fence_after();
+            }
+            for (int kb = 4 * j; kb < 4 * j + 4 && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
+          }
+        }
+        if (ok && !has_next) ok = mbar_wait(smem_u32(&dhd_bar), unit_it & 1u, abort_flag, a.err);
+        ++unit_it;
+      }
+      umma_commit_pair_mc(smem_u32(&done_bar), static_cast<uint16_t>(1u << rank));
+      mbar_wait_drain(smem_u32(&done_bar), 0, a.err);
+    }
+  } else {
+    const int q = warp & 3;
+    const int r_in = q * 32 + lane;                       // own row = TMEM lane
+    const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
+    const uint32_t box0 = box_base + (warp - 2) * kBoxesPerWarp * kBoxBytes;
+    const uint32_t acce_lead0 = mapa_shared(smem_u32(&acce_bar[0]), lead);
+    const uint32_t acce_lead1 = mapa_shared(smem_u32(&acce_bar[1]), lead);
+    const uint32_t ta_lead = mapa_shared(smem_u32(&ta_bar), lead);
+    const uint32_t tb_lead = mapa_shared(smem_u32(&tb_bar), lead);
+    const uint32_t gw_lead0 = mapa_shared(smem_u32(&gw_bar), 0);
+    const uint32_t gw_lead1 = mapa_shared(smem_u32(&gw_bar), 2);
+    // this thread's token row inside every GW buffer (K index of dW)
+    const uint32_t gw_row = (rank * 128u + static_cast<uint32_t>(r_in)) * 128u;
+    uint32_t jj = 0, nbox = 0, unit_it = 0;
+    bool ok = true;
+
+    // z (32 columns at zaddr) -> g for vocab columns vc0 .. vc0+31 of the unit:
+    // into TMEM (16 packed columns at gaddr) and into the GW buffer of the
+    // CTA that owns those columns
+    auto convert32 = [&](uint32_t zaddr, uint32_t gaddr, int vc0, float coef, float ecoef, float mu, float lseL,
+                         int lx, int nvalid, bool live) {
+      float v[32];
+      tmem_ld32(zaddr, v);
+      uint32_t w[16];
+      if (live) {
+        const int lxc = lx - vc0;
+        const int nv = nvalid - vc0;
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+          float g0, g1;
+          if constexpr (kEnt) {
+            g0 = fmaf(ecoef, v[j] - mu, coef) * ex2_approx(fmaf(v[j], kLog2e, -lseL));
+            g1 = fmaf(ecoef, v[j + 1] - mu, coef) * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+          } else {
+            g0 = coef * ex2_approx(fmaf(v[j], kLog2e, -lseL));
+            g1 = coef * ex2_approx(fmaf(v[j + 1], kLog2e, -lseL));
+          }
+          if (j == lxc) g0 -= coef;
+          if (j + 1 == lxc) g1 -= coef;
+          if (j >= nv) g0 = 0.f;
+          if (j + 1 >= nv) g1 = 0.f;
+          w[j / 2] = pack_bf16x2(g0, g1);
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) w[j] = 0u;
+      }
+      tmem_st16(gaddr, w);
+      const int owner = vc0 >> 7;                 // vocab quarter -> CTA
+      const int cq = vc0 & 127;
+      const uint32_t off = static_cast<uint32_t>((cq >> 6) * kGWBlock) + gw_row;
+      const int cc0 = (cq & 63) >> 3;             // first 16-byte chunk in the row
+      const uint32_t dst = mapa_shared(gw_base, static_cast<uint32_t>(owner)) + off;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t pos = static_cast<uint32_t>(((cc0 + i) ^ (r_in & 7)) * 16);
+        if (owner == static_cast<int>(rank))
+          st_shared_v4(gw_base + off + pos, w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+        else
+          st_shared_cluster_v4(dst + pos, w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+      }
+    };
+    // one [32 x 32] fp32 slab of this warp's rows -> reduce-add into global
+    auto drain_slab = [&](const CUtensorMap* map, const float (&v)[32], int x, int y, bool issue) {
+      const uint32_t box = box0 + (nbox & (kBoxesPerWarp - 1)) * kBoxBytes;
+      if (lane == 0) bulk_wait_group_read<kBoxesPerWarp - 1>();
+      __syncwarp();
+      write_box32(box, lane, v);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0 && issue) tma_reduce_add_2d(map, box, x, y);
+      if (lane == 0) bulk_commit_group();
+      ++nbox;
+    };
+    // one job: copy the accumulator to registers, hand it back, then drain it
+    auto drain_job = [&](const CUtensorMap* map, int x0, int y, bool issue) -> bool {
+      const uint32_t buf = jj & 1u, aph = (jj >> 1) & 1u;
+      if (!mbar_wait(smem_u32(&accf_bar[buf]), aph, abort_flag, a.err)) return false;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + lane_off + kAccCol + buf * 128;
+      float v0[32], v1[32], v2[32], v3[32];
+      tmem_ld32(taddr, v0);
+      tmem_ld32(taddr + 32, v1);
+      tmem_ld32(taddr + 64, v2);
+      tmem_ld32(taddr + 96, v3);
+      tc_fence_before();
+      mbar_arrive_cluster_relaxed(buf ? acce_lead1 : acce_lead0);
+      ++jj;
+      drain_slab(map, v0, x0, y, issue);
+      drain_slab(map, v1, x0 + 32, y, issue);
+      drain_slab(map, v2, x0 + 64, y, issue);
+      drain_slab(map, v3, x0 + 96, y, issue);
+      return true;
+    };
+
+    for (int u = quad; u < n_units && ok; u += n_quads) {
+      const QuadUnit un = quad_unit_of(u, n_tq, n_vp, a.tile_group);
+      const bool own_null = 4 * un.tq + static_cast<int>(rank) >= n_tiles;
+      const int own_row0 = tile_of(un.tq, static_cast<int>(rank)) * kTileM;
+      const int v0 = un.vp * 512;
+      const int row = own_row0 + r_in;
+      const float coef = own_null ? 0.f : a.coef[row];
+      float ecoef = 0.f, mu = 0.f;
+      if constexpr (kEnt) {
+        if (!own_null) {
+          ecoef = a.ecoef[row];
+          mu = a.mu[row];
+        }
+      }
+      const bool live = kEnt ? (coef != 0.f || ecoef != 0.f) : (coef != 0.f);
+      const float lseL = live ? a.lse[row] * kLog2e : 0.f;
+      const int lx = a.tok_p[row] - v0;
+      const int nvalid = V - v0;
+      const uint32_t zrow = tmem_base + lane_off;
+      // Z_a -> g of vocab 0..255: TMEM columns [0, 128), GW of CTAs 0 and 1
+      if (!(ok = mbar_wait_cluster(smem_u32(&zfa_bar), unit_it & 1u, abort_flag, a.err))) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c0 = 0; c0 < 256; c0 += 32)
+        convert32(zrow + kZaCol + c0, zrow + kGCol + c0 / 2, c0, coef, ecoef, mu, lseL, lx, nvalid, live);
+      fence_proxy_async_cluster();
+      tc_fence_before();
+      mbar_arrive_cluster(ta_lead);
+      mbar_arrive_cluster(gw_lead0);
+      // Z_b -> g of vocab 256..511: TMEM columns [128, 256), GW of CTAs 2 and 3
+      if (!(ok = mbar_wait_cluster(smem_u32(&zfb_bar), unit_it & 1u, abort_flag, a.err))) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int c0 = 0; c0 < 256; c0 += 32)
+        convert32(zrow + kZbCol + c0, zrow + kGCol + 128 + c0 / 2, 256 + c0, coef, ecoef, mu, lseL, lx, nvalid,
+                  live);
+      fence_proxy_async_cluster();
+      tc_fence_before();
+      mbar_arrive_cluster(tb_lead);
+      mbar_arrive_cluster(gw_lead1);
+      // dH jobs: this CTA's 128 token rows, 128 columns of H each
+      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 128, own_row0 + q * 32, !own_null);
+      // dW jobs: this CTA's 128 vocab rows (its quarter), 128 columns of H each
+      const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
+      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 128, vrow, vrow < V);
+      ++unit_it;
+    }
+    if (lane == 0) bulk_wait_group<0>();
+    __syncwarp();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();   // no CTA leaves while another may still touch its memory
+  tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    tmem_dealloc_pair(tmem_base, 512);
+  }
+}
+
+}  // namespace
+
+int lmhead_bwd_quad_max_clusters(int n_sm) {
+  static int cached = -1;
+  if (cached >= 0) return cached;
+  cudaError_t e =
+      cudaFuncSetAttribute(lmhead_bwd_quad_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  if (e != cudaSuccess) return 0;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_sm / 4 * 4, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  int n = 0;
+  e = cudaOccupancyMaxActiveClusters(&n, lmhead_bwd_quad_kernel<false>, &cfg);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    n = n_sm / 4;
+  }
+  cached = n;
+  return n;
+}
+
+cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& tm_wz, const CUtensorMap& tm_h,
+                                   const CUtensorMap& tm_w_n, const CUtensorMap& tm_dh, const CUtensorMap& tm_dw,
+                                   const BwdArgs& a, int n_sm, cudaStream_t s) {
+  const bool ent = a.ecoef != nullptr;
+  cudaError_t e = ent ? cudaFuncSetAttribute(lmhead_bwd_quad_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kSmemBytes)
+                      : cudaFuncSetAttribute(lmhead_bwd_quad_kernel<false>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  if (e != cudaSuccess) return e;
+  int clusters = lmhead_bwd_quad_max_clusters(n_sm);
+  if (clusters > n_sm / 4) clusters = n_sm / 4;
+  if (clusters < 1) clusters = 1;
+  if (ent)
+    lmhead_bwd_quad_kernel<true>
+        <<<4 * clusters, kThreads, kSmemBytes, s>>>(tm_hz, tm_wz, tm_h, tm_w_n, tm_dh, tm_dw, a);
+  else
+    lmhead_bwd_quad_kernel<false>
+        <<<4 * clusters, kThreads, kSmemBytes, s>>>(tm_hz, tm_wz, tm_h, tm_w_n, tm_dh, tm_dw, a);
+  return cudaGetLastError();
+}
+
+}  // namespace molt

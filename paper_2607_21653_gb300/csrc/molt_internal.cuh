@@ -67,6 +67,8 @@ struct BwdArgs {
   int tile_group;            // token tiles per raster group
   const float* ecoef;        // entropy-bonus coefficient per row, or nullptr
   const float* mu;           // sum_v p_v z_v per row (with ecoef)
+  float* dh32;               // [Tcap, H] fp32 dhidden accumulator
+  float* dW;                 // [V, H] fp32 dW
   unsigned* err;
 };
 
@@ -116,6 +118,10 @@ cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, 
 cudaError_t launch_lmhead_bwd_pair(const CUtensorMap& tm_h, const CUtensorMap& tm_w_z128, const CUtensorMap& tm_w_n,
                                    const CUtensorMap& tm_dh, const CUtensorMap& tm_dw, const BwdArgs& a, int n_sm,
                                    cudaStream_t s);
+// lmhead_bwd4.cu (clusters of two CTA pairs; H % 256 == 0)
+cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& tm_wz, const CUtensorMap& tm_h,
+                                   const CUtensorMap& tm_w_n, const CUtensorMap& tm_dh, const CUtensorMap& tm_dw,
+                                   const BwdArgs& a, int n_sm, cudaStream_t s);
 // lmhead_bwd.cu
 cudaError_t launch_lmhead_bwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w_z, const CUtensorMap& tm_w_n,
                               const CUtensorMap& tm_dh, const CUtensorMap& tm_dw, const BwdArgs& a, int grid,

@@ -219,6 +219,19 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo_byt
   return d;
 }
 
+// K-major operand in the 64-byte swizzle (layout 4): rows of 64 B (32 bf16
+// along K), 8-row groups SBO = 512 B apart; advancing K by 16 elements adds
+// 32 B to the start.
+__device__ __forceinline__ uint64_t sdesc_sw64(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>(512 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(4) << 61;
+  return d;
+}
+
 // Instruction descriptor for tcgen05.mma kind::f16 with bf16 A and B and an
 // fp32 accumulator: D format (bits 4-5) = F32, A/B format (bits 7-9, 10-12) =
 // BF16, A/B major (bits 15, 16: 0 = K-major, 1 = MN-major), N>>3 (bits 17-22),
