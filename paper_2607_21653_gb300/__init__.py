@@ -28,7 +28,7 @@ _CSRC = os.path.join(_PKG, "csrc")
 _INCLUDE = os.path.join(_ROOT, "include")
 _BUILD = os.path.join(_ROOT, "_build")
 _LIB = os.path.join(_PKG, "libmolt.so")
-_SOURCES = ["rows.cu", "lmhead_fwd.cu", "lmhead_bwd.cu", "lmhead_bwd2.cu", "lmhead_bwd4.cu", "api.cu", "noalloc.cu"]
+_SOURCES = ["rows.cu", "lmhead_fwd.cu", "lmhead_bwd.cu", "lmhead_bwd4.cu", "api.cu", "noalloc.cu"]
 ARCH_FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 STATUS = {

@@ -114,10 +114,6 @@ cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, 
 // lmhead_fwd.cu
 cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,
                               cudaStream_t s);
-// lmhead_bwd2.cu (CTA pairs; H % 256 == 0)
-cudaError_t launch_lmhead_bwd_pair(const CUtensorMap& tm_h, const CUtensorMap& tm_w_z128, const CUtensorMap& tm_w_n,
-                                   const CUtensorMap& tm_dh, const CUtensorMap& tm_dw, const BwdArgs& a, int n_sm,
-                                   cudaStream_t s);
 // lmhead_bwd4.cu (clusters of two CTA pairs; H % 256 == 0)
 cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& tm_wz, const CUtensorMap& tm_h,
                                    const CUtensorMap& tm_w_n, const CUtensorMap& tm_dh, const CUtensorMap& tm_dw,
