@@ -161,9 +161,13 @@ def oracle_rows_rate(w, n_rows_target_s, seed=0, max_rows=4096):
         O.policy_loss_rows(h_rows, W64, w.tokens, b, adv, w.mask, w.eps_lo, w.eps_hi, D, rows, want_dW=True)
         return time.perf_counter() - t0
 
-    probe = rng.choice(act, size=8, replace=False)
-    dt = run(probe)
-    n = int(min(max_rows, max(8, n_rows_target_s / max(dt / 8, 1e-6))))
+    # a call has a fixed cost (the V x H dW accumulator) besides its per-row
+    # cost: separate the two with probes of 8 and 64 rows
+    t8 = run(rng.choice(act, size=min(8, act.size), replace=False))
+    t64 = run(rng.choice(act, size=min(64, act.size), replace=False))
+    per_row = max((t64 - t8) / 56.0, 1e-6)
+    fixed = max(t8 - 8 * per_row, 0.0)
+    n = int(min(max_rows, max(8, (n_rows_target_s - fixed) / per_row)))
     n = max(8, (n // 8) * 8)
     rows = rng.choice(act, size=min(n, act.size), replace=False)
     dt = run(rows)
