@@ -11,7 +11,7 @@ in spans of 8-256, clip eps 0.2 / 0.28.  Inputs are synthetic and seeded
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--estimator grpo|group_mean|dr_grpo|rloo|reinforce_pp]
-                  [--objective ppo|kl_entropy_gate]
+                  [--objective ppo|kl_entropy_gate] [--deterministic]
 
 --estimator picks the advantage estimator (Sec. 4.5 list); --objective
 kl_entropy_gate adds a KL-to-reference term, an entropy bonus and the
@@ -41,7 +41,9 @@ sys.path.insert(0, ROOT)
 
 METRIC = "policy-loss fwd+bwd tokens/s on 1 GB300; % of dense bf16 tensor peak"
 KERNELS_PER_STEP = 9   # advantages, broadcast, compact, gather, forward, merge, finalize, backward, cast
-KERNELS_PER_STEP_EX = 11   # + sequence gate and loss rows (merge writes the packed row statistics)
+# the extended objective adds the loss-rows kernel (merge then writes the packed
+# row statistics) and, with a sequence gate, the gate kernel
+KERNELS_PER_STEP_EX = 10
 
 
 def load_peaks():
@@ -281,15 +283,16 @@ def run_ours(args):
     adv_tok = torch.empty(T, dtype=torch.float32, device=dev)
     dW = torch.empty(V, H, dtype=torch.float32, device=dev)
     n_active = int(w.mask.sum())
-    extended = args.objective == "kl_entropy_gate"
-    ex_opts = {}
-    if extended:
+    extended = args.objective == "kl_entropy_gate" or args.deterministic
+    ex_opts = {"deterministic": args.deterministic}
+    if args.objective == "kl_entropy_gate":
         # reference-policy log-probs: the current ones plus an independent lag;
         # one gated sequence per rollout; a band wide enough that the gate
         # rejects (and so skips) no work at this behaviour lag
         rnoise = np.random.default_rng(w.seed + 29).normal(0.0, 0.1, T).astype(np.float32)
         ex_opts = dict(kl_coef=0.01, ref_logp=(lp + torch.from_numpy(rnoise).to(dev)).contiguous(),
-                       entropy_coef=1e-3, seq_of_token=rot, gate_lo=0.5, gate_hi=2.0)
+                       entropy_coef=1e-3, seq_of_token=rot, gate_lo=0.5, gate_hi=2.0,
+                       deterministic=args.deterministic)
 
     def step(tok=tokens, msk=mask, hid=hidden, bb=b, rw=rewards, gi=gids, ro=rot, rf=None):
         if args.estimator == "grpo":
@@ -299,10 +302,11 @@ def run_ours(args):
                             out=adv_resp)
         molt.broadcast_advantages(adv_resp, ro, out=adv_tok)
         if extended:
+            opts = dict(ex_opts)
+            if "seq_of_token" in opts:
+                opts.update(seq_of_token=ro, ref_logp=opts["ref_logp"] if rf is None else rf)
             return molt.policy_loss_fwd_bwd_ex(hid, weight, tok, bb, adv_tok, msk, w.eps_lo, w.eps_hi, dW=dW,
-                                               want_token_outputs=False,
-                                               **dict(ex_opts, seq_of_token=ro,
-                                                      ref_logp=ex_opts["ref_logp"] if rf is None else rf))
+                                               want_token_outputs=False, **opts)
         return molt.policy_loss_fwd_bwd(hid, weight, tok, bb, adv_tok, msk, w.eps_lo, w.eps_hi, dW=dW,
                                         want_token_outputs=False)
 
@@ -355,7 +359,7 @@ def run_ours(args):
         copies = [(d_hid, h_hid), (d_tok, h_tok), (d_msk, h_msk), (d_b, h_b), (d_rw, h_rw), (d_gi, h_gi),
                   (d_ro, h_ro)]
         d_rf = None
-        if extended:
+        if "ref_logp" in ex_opts:
             h_rf = pin(ex_opts["ref_logp"].cpu().numpy())
             d_rf = torch.empty_like(ex_opts["ref_logp"])
             copies.append((d_rf, h_rf))
@@ -383,7 +387,7 @@ def run_ours(args):
         e2e = {"value": job_throughput(T, world, e_steps, ems), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": 4, "steps": e_steps,
                "note": "hidden, tokens, mask, behaviour log-probs, rewards, group ids and the token->rollout map "
-                       + ("(and reference log-probs) " if extended else "")
+                       + ("(and reference log-probs) " if "ref_logp" in ex_opts else "")
                        + "copied from pinned host memory every step; W stays resident; loss read back"}
 
     if rank != 0:
@@ -439,13 +443,16 @@ def run_ours(args):
                    "tensor_peak_frac_6THV": step_frac,
                    "tensor_peak_frac_6THV_of_burst": 6.0 * tp * H * V / step_s / 1e12 / peaks["bf16"],
                    "loss": loss_val, "estimator": args.estimator, "objective": args.objective,
+                   "deterministic": bool(args.deterministic),
                    **({"kl_coef": 0.01, "entropy_coef": 1e-3, "gate": [0.5, 2.0],
-                       "seq_rejected": step_stats.get("n_seq_rejected")} if extended else {})},
+                       "seq_rejected": step_stats.get("n_seq_rejected")}
+                      if args.objective == "kl_entropy_gate" else {})},
         "roofline": roofline,
         "cpu_baseline": cpu,
         "clocks": clk,
         "e2e": e2e,
-        "gpu_launches": (KERNELS_PER_STEP_EX if extended else KERNELS_PER_STEP) * args.steps,
+        "gpu_launches": ((KERNELS_PER_STEP_EX if extended else KERNELS_PER_STEP)
+                         + (1 if args.objective == "kl_entropy_gate" else 0)) * args.steps,
     }
     print(json.dumps(line), flush=True)
     if world > 1:
@@ -466,6 +473,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--estimator", default="grpo", choices=("grpo", "group_mean", "dr_grpo", "rloo", "reinforce_pp"))
     ap.add_argument("--objective", default="ppo", choices=("ppo", "kl_entropy_gate"))
+    ap.add_argument("--deterministic", action="store_true",
+                    help="bitwise-reproducible dW / dhidden (ordered reductions, one dhidden copy per band)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

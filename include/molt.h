@@ -199,6 +199,16 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
  *                 Decreasing ids set MOLT_DEV_UNSORTED_GROUPS.
  *   gate_lo, gate_hi   acceptance band of the geometric-mean ratio,
  *                 0 <= gate_lo <= gate_hi (gate_hi may be +inf)
+ *   deterministic 1: dW and dhidden are bitwise reproducible for the same inputs
+ *                 on the same device (no paper counterpart).  The backward then
+ *                 fixes the order of every partial-sum reduction: each dW row is
+ *                 reduced by one warp in a fixed unit order, and each band of
+ *                 vocabulary blocks reduces dhidden into its own fp32 copy, which
+ *                 a final pass sums in band order.  Needs H % 256 == 0
+ *                 (MOLT_ERR_UNSUPPORTED_SHAPE otherwise) and the workspace of
+ *                 molt_policy_loss_workspace_bytes_ex (one [T, H] fp32 copy per
+ *                 band, about 36 bands on a GB300).  0: reduce-adds in
+ *                 arrival order (results agree to fp32 rounding).
  */
 typedef struct {
   float kl_coef;
@@ -207,6 +217,7 @@ typedef struct {
   const int32_t* seq_of_token;
   double gate_lo;
   double gate_hi;
+  int deterministic;
 } molt_loss_options;
 
 /* molt_stats plus the extended objective's counters (device memory). */
@@ -217,11 +228,15 @@ typedef struct {
   int64_t n_seq_rejected;    /* sequences (with at least one active token) rejected */
 } molt_stats_ex;
 
+/* Workspace of molt_policy_loss_fwd_bwd_ex with these options (opts may be
+ * NULL); 0 for unsupported shapes.  Queries the current device. */
+size_t molt_policy_loss_workspace_bytes_ex(int64_t T, int64_t H, int64_t V, const molt_loss_options* opts);
+
 /*
  * molt_policy_loss_fwd_bwd with the extended objective above.  Arguments as in
  * molt_policy_loss_fwd_bwd; opts NULL (or all terms disabled) gives the same
  * results.  token_loss_out[t] = m_t l_t with the extended l_t.  The workspace
- * size is molt_policy_loss_workspace_bytes(T, H, V).
+ * size is molt_policy_loss_workspace_bytes_ex(T, H, V, opts).
  */
 molt_status molt_policy_loss_fwd_bwd_ex(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
                                         const float* behavior_logp, const float* adv, const uint8_t* mask,

@@ -118,6 +118,7 @@ def load():
         "molt_policy_loss_workspace_bytes": (SZ, [I64, I64, I64]),
         "molt_policy_loss_fwd_bwd": (I32, [P, P, P, P, P, P, I64, I64, I64, F, F, D, P, P, P, I32, P, P, P, P,
                                             P, SZ, P]),
+        "molt_policy_loss_workspace_bytes_ex": (SZ, [I64, I64, I64, P]),
         "molt_policy_loss_fwd_bwd_ex": (I32, [P, P, P, P, P, P, I64, I64, I64, F, F, D, P, P, P, P, I32, P, P,
                                                P, P, P, SZ, P]),
         "molt_set_timing_events": (None, [P, P, I32]),
@@ -401,12 +402,13 @@ def stats_dict(stats_tensor) -> dict:
 class LossOptions(ctypes.Structure):
     """molt_loss_options: KL-to-reference, entropy bonus, sequence gate."""
     _fields_ = [("kl_coef", ctypes.c_float), ("entropy_coef", ctypes.c_float), ("ref_logp", ctypes.c_void_p),
-                ("seq_of_token", ctypes.c_void_p), ("gate_lo", ctypes.c_double), ("gate_hi", ctypes.c_double)]
+                ("seq_of_token", ctypes.c_void_p), ("gate_lo", ctypes.c_double), ("gate_hi", ctypes.c_double),
+                ("deterministic", ctypes.c_int)]
 
 
 def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None, clip_lo=0.2, clip_hi=0.2,
                            denom=0.0, kl_coef=0.0, ref_logp=None, entropy_coef=0.0, seq_of_token=None,
-                           gate_lo=0.0, gate_hi=float("inf"), dW=None, accumulate_dW=False,
+                           gate_lo=0.0, gate_hi=float("inf"), deterministic=False, dW=None, accumulate_dW=False,
                            want_token_outputs=True, stream=None, workspace=None):
     """policy_loss_fwd_bwd with the extended objective
     l_t = w_t (l_pg,t + kl_coef KL_t - entropy_coef H_t) (molt_policy_loss_fwd_bwd_ex).
@@ -427,8 +429,11 @@ def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None
         ent = torch.empty(T, dtype=torch.float32, device=dev)
         tl = torch.empty(T, dtype=torch.float32, device=dev)
     opts = LossOptions(float(kl_coef), float(entropy_coef), _ptr(ref_logp, torch.float32, "ref_logp"),
-                       _ptr(seq_of_token, torch.int32, "seq_of_token"), float(gate_lo), float(gate_hi))
-    nbytes = policy_loss_workspace_bytes(T, H, V)
+                       _ptr(seq_of_token, torch.int32, "seq_of_token"), float(gate_lo), float(gate_hi),
+                       1 if deterministic else 0)
+    nbytes = int(load().molt_policy_loss_workspace_bytes_ex(T, H, V, ctypes.byref(opts)))
+    if nbytes == 0:
+        raise MoltError(2, "unsupported shape for these options")
     ws = workspace if workspace is not None else _workspace(nbytes, dev, "policy_loss")
     _check(load().molt_policy_loss_fwd_bwd_ex(
         _bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"), _ptr(tokens, torch.int32, "tokens"),

@@ -129,7 +129,7 @@ struct Layout {
   size_t lp_p, ent_p, ecoef, mu, gate_p, total;
 };
 
-Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd) {
+Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd, int dh_copies = 1) {
   const int64_t Tcap = round_tiles(T);
   const int64_t ntile = Tcap / kTileM;
   Layout L{};
@@ -153,7 +153,7 @@ Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd) {
   L.tile_flag = take(ntile * 4);
   L.tile_list = take(ntile * 4);
   L.red = take(ntile * kRedSlots * 8);
-  L.dh32 = with_bwd ? take(Tcap * H * 4) : o;
+  L.dh32 = with_bwd ? take(static_cast<size_t>(dh_copies) * Tcap * H * 4) : o;
   L.lp_p = with_bwd ? take(Tcap * 4) : o;
   L.ent_p = with_bwd ? take(Tcap * 4) : o;
   L.ecoef = with_bwd ? take(Tcap * 4) : o;
@@ -302,6 +302,8 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
     if (ex.seq && !(ex.gate_lo >= 0.0 && ex.gate_hi >= ex.gate_lo))
       return fail(MOLT_ERR_INVALID_ARG, "the gate band must satisfy 0 <= gate_lo <= gate_hi");
   }
+  const bool det = opts && opts->deterministic;
+  if (det && H % 256 != 0) return fail(MOLT_ERR_UNSUPPORTED_SHAPE, "deterministic mode needs H % 256 == 0");
   molt_status st;
   const DeviceInfo* di = device_info(&st);
   if (!di) return st;
@@ -315,7 +317,8 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   }
   const int64_t Tcap = round_tiles(T);
   const int S = choose_splits(Tcap, V, di->n_sm);
-  const Layout L = layout(T, H, V, S, true);
+  const int n_bands = det ? lmhead_bwd_quad_clusters(di->n_sm) : 1;
+  const Layout L = layout(T, H, V, S, true, n_bands);
   Scratch sc;
   MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
   const Workspace w = carve(sc.ptr, L);
@@ -330,7 +333,7 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   MOLT_TRY(make_tmap(&tm_hz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, 32, kTileM,
                      CU_TENSOR_MAP_SWIZZLE_64B));
   MOLT_TRY(make_tmap(&tm_wz32, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, 32, 128, CU_TENSOR_MAP_SWIZZLE_64B));
-  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
+  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, n_bands * Tcap, H, 32, 32));
   MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
   MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
   if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
@@ -352,7 +355,8 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   MOLT_CUDA(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, stats_ex_out, di->status, stream),
             "finalize");
   ev_stop(2, stream);
-  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
+  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(n_bands) * Tcap * H * sizeof(float), stream),
+            "memset dh32");
   if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
   BwdArgs ba{};
   ba.tok_p = w.tok_p;
@@ -365,7 +369,9 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
   ba.tile_group = pair_bwd ? 4 : 16;
   ba.dh32 = w.dh32;
-  ba.dW = dW_out;   // token tiles: 4 quads (2048 rows) or 16 tiles per raster group
+  ba.dW = dW_out;
+  ba.det_bands = det ? n_bands : 0;
+  ba.det_rows = static_cast<int>(Tcap);   // token tiles: 4 quads (2048 rows) or 16 tiles per raster group
   if (opts && ex.entropy_coef != 0.f) {
     ba.ecoef = w.ecoef;
     ba.mu = w.mu;
@@ -379,7 +385,9 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
     MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
   ev_stop(3, stream);
   ev_start(4, stream);
-  MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
+  MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), n_bands, Tcap * H, dhidden_out, di->n_sm,
+                           stream),
+            "cast dh");
   ev_stop(4, stream);
   return MOLT_OK;
 }
@@ -521,6 +529,18 @@ size_t molt_policy_loss_workspace_bytes(int64_t T, int64_t H, int64_t V) {
   const int n_sm = di ? di->n_sm : 152;
   const int64_t Tcap = round_tiles(T);
   return layout(T, H, V, choose_splits(Tcap > 0 ? Tcap : kTileM, V, n_sm), true).total;
+}
+
+size_t molt_policy_loss_workspace_bytes_ex(int64_t T, int64_t H, int64_t V, const molt_loss_options* opts) {
+  if (check_shape(T, H, V) != MOLT_OK) return 0;
+  const bool det = opts && opts->deterministic;
+  if (det && H % 256 != 0) return 0;
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  const int n_sm = di ? di->n_sm : 152;
+  const int64_t Tcap = round_tiles(T);
+  const int n_bands = det ? lmhead_bwd_quad_clusters(n_sm) : 1;
+  return layout(T, H, V, choose_splits(Tcap > 0 ? Tcap : kTileM, V, n_sm), true, n_bands).total;
 }
 
 molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,

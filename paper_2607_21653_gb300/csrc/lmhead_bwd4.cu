@@ -100,6 +100,56 @@ __device__ __forceinline__ QuadUnit quad_unit_of(int u, int n_tq, int n_vp, int 
   return {g * group + (r - vp * g_q), vp};
 }
 
+// The units one cluster processes, in order.  Raster schedule: unit u = quad,
+// quad + n_quads, ... of quad_unit_of.  Deterministic schedule (det > 0 bands,
+// one band per cluster index): band b owns vocab blocks b, b + det, ...; for
+// each block it walks every token quad in order, so each dW row is reduced by
+// one warp in a fixed sequence, and the band's dhidden contributions go to its
+// own copy of the accumulator.
+struct UnitSeq {
+  int n_tq, n_vp, n_q, group, det;
+  int u;            // raster position
+  int b, vp, tq;    // band, vocab block, token quad
+  __device__ __forceinline__ void init(int quad, int n_quads, int ntq, int nvp, int grp, int nbands) {
+    n_tq = ntq;
+    n_vp = nvp;
+    n_q = n_quads;
+    group = grp;
+    det = nbands;
+    u = quad;
+    b = quad;
+    vp = quad;
+    tq = 0;
+    settle();
+  }
+  __device__ __forceinline__ void settle() {   // skip bands without vocab blocks
+    if (det > 0)
+      while (b < det && (vp >= n_vp || n_tq == 0)) {
+        b += n_q;
+        vp = b;
+        tq = 0;
+      }
+  }
+  __device__ __forceinline__ bool valid() const {
+    return det > 0 ? (b < det && vp < n_vp && n_tq > 0) : (u < n_tq * n_vp);
+  }
+  __device__ __forceinline__ QuadUnit cur() const {
+    return det > 0 ? QuadUnit{tq, vp} : quad_unit_of(u, n_tq, n_vp, group);
+  }
+  __device__ __forceinline__ int band() const { return det > 0 ? b : 0; }
+  __device__ __forceinline__ void advance() {
+    if (det == 0) {
+      u += n_q;
+      return;
+    }
+    if (++tq == n_tq) {
+      tq = 0;
+      vp += det;
+      settle();
+    }
+  }
+};
+
 __device__ __forceinline__ void write_box32(uint32_t box, int lane, const float (&v)[32]) {
   const uint32_t rowp = box + lane * 128;
 #pragma unroll
@@ -174,7 +224,6 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   const int n_tiles = a.counts[1];
   const int n_tq = (n_tiles + 3) / 4;
   const int n_vp = (a.V + 511) / 512;
-  const int n_units = n_tq * n_vp;
   const int H = a.H, V = a.V;
   const int nZ = H / kZK;        // logit stages per vocab half (4 per dW job)
   const int nJ = H / 128;        // dH jobs = dW jobs per unit
@@ -214,22 +263,25 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         tma_load_2d_pair(sa + kStageBytes / 2, &tm_wz, fb, kb * kZK, vrow0 + static_cast<int>(prank) * 128);
         return true;
       };
-      int u = quad;
-      if (u < n_units) {
-        const QuadUnit un = quad_unit_of(u, n_tq, n_vp, a.tile_group);
+      UnitSeq seq;
+      seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_bands);
+      if (seq.valid()) {
+        const QuadUnit un = seq.cur();
         const int own_row0 = tile_of(un.tq, static_cast<int>(rank)) * kTileM;
         for (int kb = 0; kb < nZ && ok; ++kb) ok = load_z(kb, own_row0, un.vp * 512);
       }
-      for (; u < n_units && ok; u += n_quads) {
-        const QuadUnit un = quad_unit_of(u, n_tq, n_vp, a.tile_group);
+      for (; seq.valid() && ok; seq.advance()) {
+        const QuadUnit un = seq.cur();
         const int v0 = un.vp * 512;
         const int own_row0 = tile_of(un.tq, static_cast<int>(rank)) * kTileM;
         int t4[4];
         for (int k = 0; k < 4; ++k) t4[k] = tile_of(un.tq, k) * kTileM;
-        const int un_next = u + n_quads;
+        UnitSeq nseq = seq;
+        nseq.advance();
+        const bool has_next = nseq.valid();
         int n_row0 = 0, n_v0 = 0;
-        if (un_next < n_units) {
-          const QuadUnit nu = quad_unit_of(un_next, n_tq, n_vp, a.tile_group);
+        if (has_next) {
+          const QuadUnit nu = nseq.cur();
           n_row0 = tile_of(nu.tq, static_cast<int>(rank)) * kTileM;
           n_v0 = nu.vp * 512;
         }
@@ -255,7 +307,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
             if (!(ok = next_stage(sa, fb))) break;
             tma_load_2d_pair(sa, &tm_h, fb, x, t4[st]);
           }
-          if (un_next < n_units)
+          if (has_next)
             for (int kb = 4 * j; kb < 4 * j + 4 && ok; ++kb) ok = load_z(kb, n_row0, n_v0);
         }
       }
@@ -305,11 +357,14 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         tc_fence_after();
         return true;
       };
-      int u = quad;
-      if (u < n_units)
+      UnitSeq seq;
+      seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_bands);
+      if (seq.valid())
         for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
-      for (; u < n_units && ok; u += n_quads) {
-        const bool has_next = u + n_quads < n_units;
+      for (; seq.valid() && ok; seq.advance()) {
+        UnitSeq nseq = seq;
+        nseq.advance();
+        const bool has_next = nseq.valid();
         // Z_b over [128, 384): Z_a read by both CTAs and both accumulators idle
         if (!(ok = mbar_wait_cluster(smem_u32(&ta_bar), unit_it & 1u, abort_flag, a.err))) break;
         if (!(ok = acc_free(jj) && acc_free(jj + 1))) break;
@@ -469,8 +524,10 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       return true;
     };
 
-    for (int u = quad; u < n_units && ok; u += n_quads) {
-      const QuadUnit un = quad_unit_of(u, n_tq, n_vp, a.tile_group);
+    UnitSeq seq;
+    seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_bands);
+    for (; seq.valid() && ok; seq.advance()) {
+      const QuadUnit un = seq.cur();
       const bool own_null = 4 * un.tq + static_cast<int>(rank) >= n_tiles;
       const int own_row0 = tile_of(un.tq, static_cast<int>(rank)) * kTileM;
       const int v0 = un.vp * 512;
@@ -509,9 +566,21 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive_cluster(tb_lead);
       mbar_arrive_cluster(gw_lead1);
-      // dH jobs: this CTA's 128 token rows, 128 columns of H each
-      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 128, own_row0 + q * 32, !own_null);
+      // deterministic schedule: this warp's earlier reduce-adds into the same
+      // rows complete before the next ones are issued
+      auto order_drains = [&]() {
+        if (a.det_bands > 0) {
+          if (lane == 0) bulk_wait_group<0>();
+          __syncwarp();
+        }
+      };
+      // dH jobs: this CTA's 128 token rows (in the band's copy of the
+      // accumulator), 128 columns of H each
+      order_drains();
+      const int dh_row = own_row0 + q * 32 + seq.band() * a.det_rows;
+      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 128, dh_row, !own_null);
       // dW jobs: this CTA's 128 vocab rows (its quarter), 128 columns of H each
+      order_drains();
       const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
       for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 128, vrow, vrow < V);
       ++unit_it;
@@ -552,6 +621,13 @@ int lmhead_bwd_quad_max_clusters(int n_sm) {
   return n;
 }
 
+int lmhead_bwd_quad_clusters(int n_sm) {
+  int clusters = lmhead_bwd_quad_max_clusters(n_sm);
+  if (clusters > n_sm / 4) clusters = n_sm / 4;
+  if (clusters < 1) clusters = 1;
+  return clusters;
+}
+
 cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& tm_wz, const CUtensorMap& tm_h,
                                    const CUtensorMap& tm_w_n, const CUtensorMap& tm_dh, const CUtensorMap& tm_dw,
                                    const BwdArgs& a, int n_sm, cudaStream_t s) {
@@ -561,9 +637,8 @@ cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& 
                       : cudaFuncSetAttribute(lmhead_bwd_quad_kernel<false>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return e;
-  int clusters = lmhead_bwd_quad_max_clusters(n_sm);
-  if (clusters > n_sm / 4) clusters = n_sm / 4;
-  if (clusters < 1) clusters = 1;
+  const int clusters = lmhead_bwd_quad_clusters(n_sm);
+  if (a.det_bands > 0 && a.det_bands != clusters) return cudaErrorInvalidValue;
   if (ent)
     lmhead_bwd_quad_kernel<true>
         <<<4 * clusters, kThreads, kSmemBytes, s>>>(tm_hz, tm_wz, tm_h, tm_w_n, tm_dh, tm_dw, a);

@@ -69,6 +69,8 @@ struct BwdArgs {
   const float* mu;           // sum_v p_v z_v per row (with ecoef)
   float* dh32;               // [Tcap, H] fp32 dhidden accumulator
   float* dW;                 // [V, H] fp32 dW
+  int det_bands;             // 0: raster schedule; > 0: deterministic bands (one per cluster)
+  int det_rows;              // rows between the bands' dhidden accumulator copies (Tcap)
   unsigned* err;
 };
 
@@ -109,12 +111,15 @@ cudaError_t launch_merge_stats_ex(int Tcap, int V, int n_split, const Workspace&
 cudaError_t launch_seq_gate(int T, int Tcap, const LossEx& ex, const Workspace& ws, unsigned* err, cudaStream_t s);
 cudaError_t launch_loss_rows_ex(int Tcap, double denom, float clip_lo, float clip_hi, const LossEx& ex,
                                 const Workspace& ws, float* tokloss_out, cudaStream_t s);
-cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s);
+// dhidden_out[t] = bf16(sum over the n_copies accumulator copies, in copy order)
+cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, int n_copies, int64_t copy_stride, uint16_t* dh_out,
+                           int n_sm, cudaStream_t s);
 
 // lmhead_fwd.cu
 cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,
                               cudaStream_t s);
 // lmhead_bwd4.cu (clusters of two CTA pairs; H % 256 == 0)
+int lmhead_bwd_quad_clusters(int n_sm);   // clusters one launch runs (= deterministic bands)
 cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& tm_wz, const CUtensorMap& tm_h,
                                    const CUtensorMap& tm_w_n, const CUtensorMap& tm_dh, const CUtensorMap& tm_dw,
                                    const BwdArgs& a, int n_sm, cudaStream_t s);

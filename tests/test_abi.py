@@ -87,3 +87,12 @@ def test_rejects_bad_loss_options(lib):
     opts = molt.LossOptions(-1.0, 0.0, FAKE, None, 0.0, 0.0)     # negative KL weight
     args[12] = ctypes.byref(opts)
     assert molt.STATUS[lib.molt_policy_loss_fwd_bwd_ex(*args)] == "MOLT_ERR_INVALID_ARG"
+
+
+def test_workspace_query_with_options(lib):
+    plain = lib.molt_policy_loss_workspace_bytes(1000, 512, 5000)
+    assert plain > 0
+    assert lib.molt_policy_loss_workspace_bytes_ex(1000, 512, 5000, None) == plain
+    det = molt.LossOptions(0.0, 0.0, None, None, 0.0, 0.0, 1)
+    assert lib.molt_policy_loss_workspace_bytes_ex(1000, 512, 5000, ctypes.byref(det)) >= plain
+    assert lib.molt_policy_loss_workspace_bytes_ex(1000, 192, 5000, ctypes.byref(det)) == 0

@@ -218,3 +218,67 @@ def test_bad_options_rejected():
         molt.policy_loss_fwd_bwd_ex(*args, seq_of_token=t(np.zeros(64, np.int32)), gate_lo=2.0, gate_hi=1.0)
     with pytest.raises(molt.MoltError):
         molt.policy_loss_fwd_bwd_ex(*args, entropy_coef=float("nan"))
+
+
+# ----------------------------------------------------------- deterministic mode
+DET_SHAPES = [(1000, 256, 5000), (513, 512, 4133), (640, 768, 2304), (1, 256, 7)]
+
+
+@pytest.mark.parametrize("T,H,V", DET_SHAPES)
+def test_deterministic_mode_is_bitwise_reproducible(T, H, V):
+    rng = np.random.default_rng(T + 7 * H)
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.3, w_std=0.05)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.28, T + 3)
+    runs = []
+    for _ in range(3):
+        o = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28, deterministic=True)
+        torch.cuda.synchronize()
+        assert molt.device_status() == 0
+        runs.append({k: np_(o[k]).copy() for k in ("loss", "dhidden", "dW", "logp", "token_loss")})
+    for r in runs[1:]:
+        for k in r:
+            np.testing.assert_array_equal(r[k].view(np.uint8), runs[0][k].view(np.uint8), err_msg=k)
+    ref = O.policy_loss_ex(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), m, 0.2, 0.28)
+    assert_grad_close(runs[0]["dhidden"], ref["dH"], "dhidden (deterministic)")
+    assert_grad_close(runs[0]["dW"], ref["dW"], "dW (deterministic)")
+    assert abs(float(runs[0]["loss"][0]) - ref["loss"]) <= LOSS_RTOL * max(
+        abs(ref["loss"]), float(np.abs(ref["ratio"] * adv)[m != 0].sum() / ref["denom"]))
+
+
+def test_deterministic_mode_accumulates_and_combines_with_extended_terms():
+    rng = np.random.default_rng(21)
+    lengths = [300, 1, 64, 400, 35]
+    h, W, x, m, seq, b, _ = _gated_problem(rng, 512, 3000, lengths)
+    T = seq.size
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    lp, _ = O.token_logprobs(O.widen_bf16(h), O.widen_bf16(W), x, None)
+    ref_logp = (lp + rng.normal(0, 0.3, T)).astype(np.float32)
+    kw = dict(kl_coef=0.1, ref_logp=ref_logp, entropy_coef=0.02, seq_of_token=seq, gate_lo=0.6, gate_hi=1.5)
+    dW0 = (0.01 * rng.standard_normal((3000, 512))).astype(np.float32)
+    outs = []
+    for _ in range(2):
+        dW = t(dW0.copy())
+        o = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.3, 0.3, dW=dW,
+                                        accumulate_dW=True, deterministic=True,
+                                        **{k: (t(v) if isinstance(v, np.ndarray) else v) for k, v in kw.items()})
+        torch.cuda.synchronize()
+        assert molt.device_status() == 0
+        outs.append((np_(o["dW"]).copy(), np_(o["dhidden"]).copy()))
+    np.testing.assert_array_equal(outs[0][0].view(np.uint32), outs[1][0].view(np.uint32))
+    np.testing.assert_array_equal(outs[0][1].view(np.uint16), outs[1][1].view(np.uint16))
+    ref = O.policy_loss_ex(O.widen_bf16(h), O.widen_bf16(W), x, b.astype(np.float64), adv.astype(np.float64), m,
+                           0.3, 0.3, **kw)
+    assert_grad_close(outs[0][0] - dW0, ref["dW"], "dW (accumulated, deterministic)")
+    assert_grad_close(outs[0][1], ref["dH"], "dhidden (deterministic, extended terms)")
+
+
+def test_deterministic_mode_needs_h_multiple_of_256():
+    rng = np.random.default_rng(4)
+    h, W, x, m = random_problem(rng, 64, 192, 300)
+    z = np.zeros(64, np.float32)
+    with pytest.raises(molt.MoltError):
+        molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(z), t(z), t(m), 0.2, 0.2, deterministic=True)
