@@ -440,7 +440,9 @@ def run_ours(args):
         "config": {"workload": workload_desc(w), "global_batch_tokens": world * T, "active_tokens": n_active,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 (W 1.24 GB); no flush",
+                   "active_tokens_per_s": job_throughput(n_active, world, args.steps, ms),
                    "tensor_peak_frac_6THV": step_frac,
+                   "tensor_peak_frac_8THV": step_frac * 8.0 / 6.0,
                    "tensor_peak_frac_6THV_of_burst": 6.0 * tp * H * V / step_s / 1e12 / peaks["bf16"],
                    "loss": loss_val, "estimator": args.estimator, "objective": args.objective,
                    "deterministic": bool(args.deterministic),
@@ -463,7 +465,7 @@ def run_ours(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", default="large_vocab")
