@@ -165,3 +165,21 @@ def test_fullsize_token_logprobs():
     assert np.abs(lp[rows] - lp_ref).max() <= LOGP_ATOL
     assert np.abs(ent[rows] - ent_ref).max() <= LOGP_ATOL
     assert (lp[w.mask == 0] == 0).all()
+
+
+def test_fullsize_deterministic_mode():
+    """Deterministic backward at the benchmark size: two calls agree bit for bit
+    on dW and dhidden, and sampled rows match the oracle."""
+    w, rows, b, adv, D, _, ref, hid, Wd = _run_fullsize("large_vocab")
+    outs = []
+    for _ in range(2):
+        o = molt.policy_loss_fwd_bwd_ex(hid, Wd, t(w.tokens), t(b), t(adv.astype(np.float32)), t(w.mask),
+                                        w.eps_lo, w.eps_hi, deterministic=True)
+        torch.cuda.synchronize()
+        assert molt.device_status() == 0
+        outs.append(o)
+    assert torch.equal(outs[0]["dW"].view(torch.int32), outs[1]["dW"].view(torch.int32))
+    assert torch.equal(outs[0]["dhidden"].view(torch.int16), outs[1]["dhidden"].view(torch.int16))
+    assert float(outs[0]["loss"].item()) == float(outs[1]["loss"].item())
+    dh = outs[0]["dhidden"]
+    assert_grad_close(np_(dh[torch.from_numpy(rows).to(dh.device)]), ref["dH"], "dhidden (deterministic, sampled)")
