@@ -471,7 +471,7 @@ def main():
     ap.add_argument("--workload", default="large_vocab")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--estimator", default="grpo", choices=("grpo", "group_mean", "dr_grpo", "rloo", "reinforce_pp"))
     ap.add_argument("--objective", default="ppo", choices=("ppo", "kl_entropy_gate"))
