@@ -1,0 +1,85 @@
+"""Seeded shape fuzzing of the policy-loss call against the fp64 oracle: token
+counts that leave 1-3 tiles of the last quad empty, vocabularies with ragged
+512-column blocks, H from 256 (two jobs per unit) upward, both the cluster
+backward (H % 256 == 0) and the single-CTA one, the deterministic schedule, and
+caller-provided workspaces."""
+import ctypes
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import paper_2607_21653_gb300 as molt  # noqa: E402
+from oracle import molt_oracle as O  # noqa: E402
+from workloads import random_problem  # noqa: E402
+
+from parity import LOGP_ATOL, assert_grad_close, assert_loss_close, behavior_from_oracle, bf, np_, t  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    molt.build()
+    molt.load()
+
+
+def _cases():
+    rng = np.random.default_rng(2607)
+    out = []
+    for i in range(10):
+        H = int(rng.choice([256, 512, 768, 1024, 1280, 320]))
+        T = int(rng.integers(1, 1800))
+        V = int(rng.integers(1, 7000))
+        out.append((i, T, H, V, bool(i % 3 == 0) and H % 256 == 0))
+    return out
+
+
+@pytest.mark.parametrize("i,T,H,V,det", _cases())
+def test_random_shapes(i, T, H, V, det):
+    rng = np.random.default_rng(100 + i)
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=float(rng.uniform(0.0, 0.6)), w_std=0.05)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.28, 7 + i)
+    if det:
+        out = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28, deterministic=True)
+    else:
+        out = molt.policy_loss_fwd_bwd(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    ref = O.policy_loss(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), m, 0.2, 0.28)
+    ref["_adv"] = adv.astype(np.float64)
+    assert_loss_close(float(out["loss"].item()), ref)
+    assert np.abs(np_(out["logp"]) - ref["logp"]).max() <= LOGP_ATOL
+    dh = np_(out["dhidden"])
+    assert (dh[m == 0] == 0).all()
+    assert_grad_close(dh, ref["dH"], f"dhidden case {i}")
+    assert_grad_close(np_(out["dW"]), ref["dW"], f"dW case {i}")
+
+
+def test_caller_workspace_and_too_small_workspace():
+    rng = np.random.default_rng(3)
+    T, H, V = 700, 512, 3000
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    b = behavior_from_oracle(O.widen_bf16(h), O.widen_bf16(W), x, 0.3, 0.2, 0.2, 5)
+    opts = molt.LossOptions(0.0, 0.0, None, None, 0.0, 0.0, 1)
+    need = molt.load().molt_policy_loss_workspace_bytes_ex(T, H, V, ctypes.byref(opts))
+    assert need > molt.load().molt_policy_loss_workspace_bytes(T, H, V)
+    ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+    a = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2, deterministic=True,
+                                    workspace=ws)
+    c = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2, deterministic=True)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    assert torch.equal(a["dW"].view(torch.int32), c["dW"].view(torch.int32))
+    small = torch.empty(need - 4096, dtype=torch.uint8, device="cuda")
+    with pytest.raises(molt.MoltError):
+        molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2, deterministic=True,
+                                    workspace=small)
