@@ -176,6 +176,33 @@ def oracle_rows_rate(w, n_rows_target_s, seed=0, max_rows=4096):
     return len(rows) / dt, len(rows), dt
 
 
+def oracle_tiny_whole_rate():
+    """Oracle tokens/s on the whole tiny workload (T=512, H=256, V=4096): the
+    full forward and backward of every row."""
+    from oracle import molt_oracle as O
+    from workloads import make_workload
+    w = make_workload("tiny")
+    rng = np.random.default_rng(0)
+    adv = rng.standard_normal(w.T)
+    b = rng.normal(-np.log(w.V) - 1.0, 1.0, w.T)
+    h64, W64 = O.widen_bf16(w.hidden), O.widen_bf16(w.weight)
+    t0 = time.perf_counter()
+    O.policy_loss(h64, W64, w.tokens, b, adv, w.mask, w.eps_lo, w.eps_hi)
+    return w.T / (time.perf_counter() - t0)
+
+
+def oracle_single_thread_rate():
+    """oracle_tiny_whole_rate in a child process whose BLAS runs one thread."""
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    code = "import bench; print(bench.oracle_tiny_whole_rate())"
+    try:
+        r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, env=env, capture_output=True, text=True,
+                           timeout=120)
+        return float(r.stdout.strip().splitlines()[-1])
+    except Exception:   # the extra figure is optional; the line stays valid without it
+        return None
+
+
 def run_reference(args):
     """--impl reference: the fp64 oracle on the host cores, per step a bounded
     sample of rows of the same workload."""
@@ -422,7 +449,9 @@ def run_ours(args):
         rate, nrows, secs = oracle_rows_rate(w, args.cpu_seconds)
         cpu = {"value": rate, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": f"{nrows} random active rows of the same batch (forward, dhidden rows, dW contribution), "
-                         f"{secs:.1f} s, numpy fp64 BLAS on all host cores"}
+                         f"{secs:.1f} s, numpy fp64 BLAS on all host cores",
+               "tiny_whole_tokens_per_s": oracle_tiny_whole_rate(),
+               "tiny_whole_single_thread_tokens_per_s": oracle_single_thread_rate()}
 
     line = {
         "metric": METRIC,
