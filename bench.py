@@ -163,13 +163,10 @@ def oracle_rows_rate(w, n_rows_target_s, seed=0, max_rows=4096):
         O.policy_loss_rows(h_rows, W64, w.tokens, b, adv, w.mask, w.eps_lo, w.eps_hi, D, rows, want_dW=True)
         return time.perf_counter() - t0
 
-    # a call has a fixed cost (the V x H dW accumulator) besides its per-row
-    # cost: separate the two with probes of 8 and 64 rows
-    t8 = run(rng.choice(act, size=min(8, act.size), replace=False))
+    # size the sample from a 64-row probe, charging the call's fixed cost (the
+    # V x H dW accumulator) to its rows: this never overshoots the target
     t64 = run(rng.choice(act, size=min(64, act.size), replace=False))
-    per_row = max((t64 - t8) / 56.0, 1e-6)
-    fixed = max(t8 - 8 * per_row, 0.0)
-    n = int(min(max_rows, max(8, (n_rows_target_s - fixed) / per_row)))
+    n = int(min(max_rows, max(8, n_rows_target_s * 64 / max(t64, 1e-6))))
     n = max(8, (n // 8) * 8)
     rows = rng.choice(act, size=min(n, act.size), replace=False)
     dt = run(rows)
@@ -379,33 +376,54 @@ def run_ours(args):
         h_hid = pin(w.hidden.view(np.int16))
         h_tok, h_msk, h_b = pin(w.tokens), pin(w.mask), pin(b.cpu().numpy())
         h_rw, h_gi, h_ro = pin(w.rewards), pin(w.group_ids), pin(w.resp_of_token)
-        d_hid = torch.empty(T, H, dtype=torch.int16, device=dev)
-        d_tok, d_msk, d_b = torch.empty_like(tokens), torch.empty_like(mask), torch.empty_like(b)
-        d_rw, d_gi, d_ro = torch.empty_like(rewards), torch.empty_like(gids), torch.empty_like(rot)
+        h_rf = pin(ex_opts["ref_logp"].cpu().numpy()) if "ref_logp" in ex_opts else None
         h_loss = torch.empty(1, dtype=torch.float32).pin_memory()
-        copies = [(d_hid, h_hid), (d_tok, h_tok), (d_msk, h_msk), (d_b, h_b), (d_rw, h_rw), (d_gi, h_gi),
-                  (d_ro, h_ro)]
-        d_rf = None
-        if "ref_logp" in ex_opts:
-            h_rf = pin(ex_opts["ref_logp"].cpu().numpy())
-            d_rf = torch.empty_like(ex_opts["ref_logp"])
-            copies.append((d_rf, h_rf))
-        h2d = sum(src.numel() * src.element_size() for _, src in copies)
-        e_steps = max(1, args.steps // 2)
-        for dst, src in copies:
-            dst.copy_(src)
+        # two sets of device inputs: step k computes from set k % 2 while the
+        # host-to-device copies of step k + 1 fill the other set on a copy stream
+        sets = []
         for _ in range(2):
-            o = step(d_tok, d_msk, d_hid.view(torch.bfloat16), d_b, d_rw, d_gi, d_ro, d_rf)
+            d_hid = torch.empty(T, H, dtype=torch.int16, device=dev)
+            d_tok, d_msk, d_b = torch.empty_like(tokens), torch.empty_like(mask), torch.empty_like(b)
+            d_rw, d_gi, d_ro = torch.empty_like(rewards), torch.empty_like(gids), torch.empty_like(rot)
+            d_rf = torch.empty_like(ex_opts["ref_logp"]) if h_rf is not None else None
+            cps = [(d_hid, h_hid), (d_tok, h_tok), (d_msk, h_msk), (d_b, h_b), (d_rw, h_rw), (d_gi, h_gi),
+                   (d_ro, h_ro)] + ([(d_rf, h_rf)] if h_rf is not None else [])
+            sets.append((cps, (d_tok, d_msk, d_hid.view(torch.bfloat16), d_b, d_rw, d_gi, d_ro, d_rf)))
+        h2d = sum(src.numel() * src.element_size() for _, src in sets[0][0])
+        e_steps = max(2, args.steps // 2)
+        comp = torch.cuda.current_stream(dev)
+        copy_stream = torch.cuda.Stream(device=dev)
+        copied = [torch.cuda.Event() for _ in range(2)]
+        freed = [torch.cuda.Event() for _ in range(2)]
+        go = torch.cuda.Event()
+
+        def issue_copies(k):
+            with torch.cuda.stream(copy_stream):
+                copy_stream.wait_event(freed[k % 2] if k >= 2 else go)   # set free, timed region open
+                for dst, src in sets[k % 2][0]:
+                    dst.copy_(src, non_blocking=True)
+                copied[k % 2].record(copy_stream)
+
+        def run_e2e(n):
+            go.record(comp)
+            issue_copies(0)
+            out = None
+            for k in range(n):
+                if k + 1 < n:
+                    issue_copies(k + 1)
+                comp.wait_event(copied[k % 2])
+                out = step(*sets[k % 2][1])
+                freed[k % 2].record(comp)
+                h_loss.copy_(out["loss"], non_blocking=True)
+            return out
+
+        run_e2e(2)
         torch.cuda.synchronize()
         barrier()
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
-        for _ in range(e_steps):
-            for dst, src in copies:
-                dst.copy_(src, non_blocking=True)
-            o = step(d_tok, d_msk, d_hid.view(torch.bfloat16), d_b, d_rw, d_gi, d_ro, d_rf)
-            h_loss.copy_(o["loss"], non_blocking=True)
+        run_e2e(e_steps)
         e1.record()
         torch.cuda.synchronize()
         assert molt.device_status() == 0
@@ -415,7 +433,8 @@ def run_ours(args):
                "d2h_bytes_per_step": 4, "steps": e_steps,
                "note": "hidden, tokens, mask, behaviour log-probs, rewards, group ids and the token->rollout map "
                        + ("(and reference log-probs) " if "ref_logp" in ex_opts else "")
-                       + "copied from pinned host memory every step; W stays resident; loss read back"}
+                       + "copied from pinned host memory every step, on a copy stream into one of two device "
+                         "input sets while the previous step computes; W stays resident; loss read back every step"}
 
     if rank != 0:
         if world > 1:
