@@ -79,9 +79,11 @@ def recorded_traffic(kernel):
     return None
 
 
-def workload_desc(w):
+def workload_desc(w, microbatch=0):
+    window = w.extra.get("window_tokens")
     return (f"{w.name}: T={w.T}, H={w.H}, V={w.V}, bf16, "
-            f"{100 * (1 - w.mask.mean()):.0f}% masked in spans, clip {w.eps_lo}/{w.eps_hi}")
+            f"{100 * (1 - w.mask.mean()):.0f}% masked in spans, clip {w.eps_lo}/{w.eps_hi}"
+            + (f", microbatch {microbatch} of a {window}-token window" if window else ""))
 
 
 # ------------------------------------------------------------------ clocks
@@ -200,6 +202,15 @@ def oracle_single_thread_rate():
         return None
 
 
+def microbatch_of(args):
+    """Microbatch of a windowed workload: the ragged window's first one holds only
+    its two constant-reward groups (every advantage 0, no gradient), so it
+    defaults to microbatch 1."""
+    if args.microbatch is not None:
+        return args.microbatch
+    return 1 if args.workload == "ragged" else 0
+
+
 def run_reference(args):
     """--impl reference: the fp64 oracle on the host cores, per step a bounded
     sample of rows of the same workload."""
@@ -207,7 +218,7 @@ def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    w = make_workload(args.workload)
+    w = make_workload(args.workload, microbatch=microbatch_of(args))
     from oracle import molt_oracle as O
     rng = np.random.default_rng(1)
     act = np.nonzero(w.mask)[0]
@@ -235,7 +246,7 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": workload_desc(w), "sample": f"{rows_per_step} random active rows per step"},
+        "config": {"workload": workload_desc(w, microbatch_of(args)), "sample": f"{rows_per_step} random active rows per step"},
         "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
                          "sample": f"{rows_per_step} active rows per step (forward, dhidden rows, dW contribution)"},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -286,7 +297,7 @@ def run_ours(args):
     molt.load()
     peaks = load_peaks()
 
-    w = make_workload(args.workload, seed=rank_seed(None, rank, world))
+    w = make_workload(args.workload, seed=rank_seed(None, rank, world), microbatch=microbatch_of(args))
     T, H, V = w.T, w.H, w.V
 
     def bf(bits):
@@ -485,7 +496,7 @@ def run_ours(args):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
-        "config": {"workload": workload_desc(w), "global_batch_tokens": world * T, "active_tokens": n_active,
+        "config": {"workload": workload_desc(w, microbatch_of(args)), "global_batch_tokens": world * T, "active_tokens": n_active,
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 (W 1.24 GB); no flush",
                    "active_tokens_per_s": job_throughput(n_active, world, args.steps, ms),
@@ -523,6 +534,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--estimator", default="grpo", choices=("grpo", "group_mean", "dr_grpo", "rloo", "reinforce_pp"))
     ap.add_argument("--objective", default="ppo", choices=("ppo", "kl_entropy_gate"))
+    ap.add_argument("--microbatch", type=int, default=None,
+                    help="microbatch of a windowed workload (ragged: default 1)")
     ap.add_argument("--deterministic", action="store_true",
                     help="bitwise-reproducible dW / dhidden (ordered reductions, one dhidden copy per band)")
     args = ap.parse_args()
