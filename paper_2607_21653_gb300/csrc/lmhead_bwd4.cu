@@ -53,6 +53,7 @@
 // Roles per CTA (192 threads): warp 0 TMA producer (each CTA loads its half of
 // every operand; bytes complete on the pair leader's barrier), warp 1 MMA issuer
 // (pair leaders only) and TMEM owner, warps 2-5 epilogue.
+#include <atomic>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -602,8 +603,13 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
 }  // namespace
 
 int lmhead_bwd_quad_max_clusters(int n_sm) {
-  static int cached = -1;
-  if (cached >= 0) return cached;
+  // per device: the number of 4-CTA clusters that fit at this kernel's
+  // shared-memory size (cached as value + 1; 0 = not queried yet)
+  static std::atomic<int> cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  const int c = cache[dev & 63].load(std::memory_order_acquire);
+  if (c > 0) return c - 1;
   cudaError_t e =
       cudaFuncSetAttribute(lmhead_bwd_quad_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return 0;
@@ -617,7 +623,7 @@ int lmhead_bwd_quad_max_clusters(int n_sm) {
     cudaGetLastError();
     n = n_sm / 4;
   }
-  cached = n;
+  cache[dev & 63].store(n + 1, std::memory_order_release);
   return n;
 }
 

@@ -17,6 +17,7 @@
 //   warp 1      MMA issuer (one lane): tcgen05.mma kind::f16, M=128 N=256 K=16,
 //               double-buffered accumulators (2 x 256 TMEM columns)
 //   warps 2-5   epilogue: each thread owns one TMEM lane = one token row
+#include <atomic>
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -285,11 +286,16 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,
                               cudaStream_t s) {
-  static bool attr_set = false;   // set once per process; same value for every device
-  if (!attr_set) {
-    cudaError_t e = cudaFuncSetAttribute(lmhead_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+  // the shared-memory attribute is per device: set it on each device once
+  static std::atomic<unsigned long long> attr_set{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const unsigned long long bit = 1ull << (dev & 63);
+  if ((attr_set.load(std::memory_order_acquire) & bit) == 0) {
+    e = cudaFuncSetAttribute(lmhead_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    attr_set.fetch_or(bit, std::memory_order_release);
   }
   lmhead_fwd_kernel<<<grid, kThreads, kSmemBytes, s>>>(tm_h, tm_w, a);
   return cudaGetLastError();
