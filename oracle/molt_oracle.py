@@ -52,7 +52,8 @@ autograd gradient of advantage-weighted cross-entropy, clipped rows having zero
 gradient, special clip values, finite differences of the loss, microbatch-split
 invariance of Eq. 2 and segment-split invariance of the advantages; for the
 extended objective, torch autograd of PPO + k3 KL - entropy bonus, the
-reduction to the plain loss, and hand-built gate cases.
+reduction to the plain loss, hand-built gate cases, and policy_loss_ex_rows as
+an exact slice of policy_loss_ex.
 """
 from __future__ import annotations
 
@@ -63,7 +64,7 @@ import numpy as np
 __all__ = [
     "widen_bf16", "group_advantages", "advantages", "ESTIMATORS", "broadcast_advantages", "logits_rows",
     "row_softmax_stats", "token_logprobs", "policy_loss", "policy_loss_rows",
-    "clip_decision", "surrogate", "policy_loss_ex", "sequence_gate",
+    "clip_decision", "surrogate", "policy_loss_ex", "sequence_gate", "policy_loss_ex_rows",
 ]
 
 DEFAULT_ADV_EPS = 1e-6
@@ -421,4 +422,53 @@ def policy_loss_ex(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, behavi
         out["kl"][t] = kl
         out["clipped"][t] = clipped
     out.update(loss=float(out["token_loss"].sum() / D), denom=D, dH=dH, dW=dW)
+    return out
+
+
+def policy_loss_ex_rows(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, behavior_logp: np.ndarray,
+                        adv: np.ndarray, mask: np.ndarray, eps_lo: float, eps_hi: float, denom: float,
+                        rows: np.ndarray, kl_coef: float = 0.0, ref_logp: np.ndarray | None = None,
+                        entropy_coef: float = 0.0, gate_w: np.ndarray | None = None, block: int = 64):
+    """policy_loss_ex restricted to the given rows, with the sequence-gate
+    weights w_t supplied (gate_w[t] for every token t; None = all 1): the gate
+    needs every token of a sequence, the per-row terms only the row itself.
+    Returns logp, entropy, ratio, kl, token_loss (m w l), coef and dH for the
+    rows, in their order."""
+    rows = np.asarray(rows)
+    n = rows.shape[0]
+    out = {k: np.zeros(n) for k in ("logp", "entropy", "ratio", "kl", "token_loss", "coef")}
+    out["dH"] = np.zeros((n, hidden.shape[1]))
+    m_all = np.asarray(mask).astype(np.float64)
+    w_all = np.ones(len(m_all)) if gate_w is None else np.asarray(gate_w, dtype=np.float64)
+    for b0 in range(0, n, block):
+        pos = np.arange(b0, min(n, b0 + block))
+        t = rows[pos]
+        act = m_all[t] != 0
+        if not act.any():
+            continue
+        pos, t = pos[act], t[act]
+        x = np.asarray(tokens)[t]
+        z = logits_rows(hidden[t], W)
+        lse, logp, ent, p = row_softmax_stats(z, x)
+        rho = np.exp(logp - np.asarray(behavior_logp, dtype=np.float64)[t])
+        l_pg, c, _ = surrogate(rho, np.asarray(adv, dtype=np.float64)[t], eps_lo, eps_hi)
+        if ref_logp is not None and kl_coef != 0.0:
+            r = np.asarray(ref_logp, dtype=np.float64)[t] - logp
+            kl, c_kl = np.exp(r) - r - 1.0, kl_coef * (np.exp(r) - 1.0)
+        else:
+            kl, c_kl = np.zeros_like(logp), np.zeros_like(logp)
+        wt = w_all[t]
+        coef = wt * (c + c_kl) / denom
+        g = coef[:, None] * p
+        g[np.arange(t.shape[0]), x] -= coef
+        if entropy_coef != 0.0:
+            mu = (p * z).sum(axis=1)
+            g += (wt * entropy_coef / denom)[:, None] * p * (z - mu[:, None])
+        out["logp"][pos] = logp
+        out["entropy"][pos] = ent
+        out["ratio"][pos] = rho
+        out["kl"][pos] = kl
+        out["token_loss"][pos] = wt * (l_pg + kl_coef * kl - entropy_coef * ent)
+        out["coef"][pos] = coef
+        out["dH"][pos] = g @ W
     return out

@@ -190,3 +190,52 @@ def test_fullsize_deterministic_mode():
     assert float(outs[0]["loss"].item()) == float(outs[1]["loss"].item())
     dh = outs[0]["dhidden"]
     assert_grad_close(np_(dh[torch.from_numpy(rows).to(dh.device)]), ref["dH"], "dhidden (deterministic, sampled)")
+
+
+def test_fullsize_extended_objective():
+    """KL, entropy bonus and sequence gate at the benchmark size.  One sequence
+    per response; each sequence's mean log-ratio is placed (from the library's
+    own log-probs) either inside the gate band or 0.3+ outside it, so every gate
+    decision is fixed by construction; sampled rows are checked against the
+    oracle with those gate weights, and the rejection counts exactly."""
+    w = make_workload("large_vocab")
+    rng = np.random.default_rng(99)
+    W64 = _w64(w)
+    rows = _sample_rows(w, rng)
+    h_rows64 = np.zeros((w.T, w.H))
+    h_rows64[rows] = O.widen_bf16(w.hidden[rows])
+    hid, Wd = bf(w.hidden), bf(w.weight)
+    lp_dev, _ = molt.token_logprobs(hid, Wd, t(w.tokens), None)
+    lp = np_(lp_dev).astype(np.float64)
+    seq = w.resp_of_token.astype(np.int32)
+    assert (np.diff(seq) >= 0).all()
+    n_seq = int(seq.max()) + 1
+    act = w.mask != 0
+    targets = rng.choice([-0.05, 0.0, 0.05, 0.8, -0.9], size=n_seq)
+    noise = rng.uniform(-0.04, 0.04, w.T)
+    cnt = np.bincount(seq, weights=act.astype(np.float64), minlength=n_seq)
+    mean_noise = np.bincount(seq, weights=noise * act, minlength=n_seq) / np.maximum(cnt, 1)
+    lr = targets[seq] + noise - mean_noise[seq]
+    b = (lp - lr).astype(np.float32)
+    ref_logp = (lp + rng.normal(0, 0.3, w.T)).astype(np.float32)
+    adv = O.broadcast_advantages(O.group_advantages(w.rewards, w.group_ids), w.resp_of_token).astype(np.float32)
+    lo, hi = 0.6, 1.5
+    kept = (np.log(lo) <= targets) & (targets <= np.log(hi))
+    gate_w = np.where(kept[seq], 1.0, 0.0)
+    out = molt.policy_loss_fwd_bwd_ex(hid, Wd, t(w.tokens), t(b), t(adv), t(w.mask), w.eps_lo, w.eps_hi,
+                                      kl_coef=0.05, ref_logp=t(ref_logp), entropy_coef=0.01,
+                                      seq_of_token=t(seq), gate_lo=lo, gate_hi=hi)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    D = float(act.sum())
+    ref = O.policy_loss_ex_rows(h_rows64, W64, w.tokens, b.astype(np.float64), adv.astype(np.float64), w.mask,
+                                w.eps_lo, w.eps_hi, D, rows, kl_coef=0.05, ref_logp=ref_logp, entropy_coef=0.01,
+                                gate_w=gate_w)
+    assert np.abs(np_(out["logp"])[rows] - ref["logp"]).max() <= LOGP_ATOL
+    np.testing.assert_allclose(np_(out["token_loss"])[rows], ref["token_loss"], rtol=5e-3, atol=2e-5)
+    dh = out["dhidden"]
+    assert_grad_close(np_(dh[torch.from_numpy(rows).to(dh.device)]), ref["dH"], "dhidden (extended, sampled)")
+    st = molt.stats_dict(out["stats"])
+    live_seq = cnt > 0
+    assert st["n_seq_rejected"] == int((~kept & live_seq).sum())
+    assert st["n_tokens_rejected"] == int((act & ~kept[seq]).sum())

@@ -387,3 +387,16 @@ def test_sequence_gate_rejects_without_renormalising():
     m3 = m.copy()
     m3[8:] = 0
     np.testing.assert_array_equal(O.sequence_gate(lr, seq, m3, 0.5, 1.5)[8:], 1.0)
+
+
+def test_ex_rows_is_a_slice_of_the_full_extended_loss():
+    h, W, x, m, adv, b, ref = _ex_problem(4, T=20, H=12, V=30)
+    seq = np.repeat(np.arange(4), 5).astype(np.int32)
+    full = O.policy_loss_ex(h, W, x, b, adv, m, 0.2, 0.28, kl_coef=0.2, ref_logp=ref, entropy_coef=0.05,
+                            seq_of_token=seq, gate_lo=0.8, gate_hi=1.25)
+    rows = np.array([17, 3, 0, 11, 8])
+    part = O.policy_loss_ex_rows(h, W, x, b, adv, m, 0.2, 0.28, full["denom"], rows, kl_coef=0.2, ref_logp=ref,
+                                 entropy_coef=0.05, gate_w=full["gate"])
+    for k in ("logp", "token_loss", "coef"):
+        np.testing.assert_allclose(part[k], full[k][rows], rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(part["dH"], full["dH"][rows], rtol=1e-12, atol=1e-15)
