@@ -54,7 +54,7 @@ def test_group_advantages_edge_cases():
 
 
 @pytest.mark.parametrize("estimator", ["grpo", "group_mean", "dr_grpo", "rloo", "reinforce_pp"])
-@pytest.mark.parametrize("name", ["tiny", "mid", "ragged"])
+@pytest.mark.parametrize("name", ["tiny", "mid", "large_vocab", "long_traj", "ragged"])
 def test_estimators_bit_exact(name, estimator):
     w = make_workload(name, with_tensors=False)
     ref = O.advantages(w.rewards, w.group_ids, estimator)
