@@ -235,10 +235,12 @@ def _stream(stream=None):
 _ws_cache: dict = {}
 
 
-def _workspace(nbytes: int, device, key: str):
-    """Workspace buffer from the torch caching allocator, reused per (device, key)."""
+def _workspace(nbytes: int, device, key: str, stream=None):
+    """Workspace buffer from the torch caching allocator, reused per (device,
+    call kind, stream): calls on one stream run in order and can share it, calls
+    on different streams may overlap and get their own."""
     torch = _torch()
-    k = (str(device), key)
+    k = (str(device), key, _stream(stream))
     buf = _ws_cache.get(k)
     if buf is None or buf.numel() < nbytes:
         buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
@@ -321,7 +323,7 @@ def token_logprobs(hidden, weight, tokens, mask=None, want_entropy=True, stream=
     logp = torch.empty(T, dtype=torch.float32, device=hidden.device)
     ent = torch.empty(T, dtype=torch.float32, device=hidden.device) if want_entropy else None
     nbytes = token_logprobs_workspace_bytes(T, H, V)
-    ws = workspace if workspace is not None else _workspace(nbytes, hidden.device, "logprobs")
+    ws = workspace if workspace is not None else _workspace(nbytes, hidden.device, "logprobs", stream)
     _check(load().molt_token_logprobs_fwd(_bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"),
                                           _ptr(tokens, torch.int32, "tokens"), _ptr(mask, torch.uint8, "mask"),
                                           T, H, V, _ptr(logp), _ptr(ent), ws.data_ptr(), ws.numel(),
@@ -370,7 +372,7 @@ def policy_loss_fwd_bwd(hidden, weight, tokens, behavior_logp, adv, mask=None, c
         ent = torch.empty(T, dtype=torch.float32, device=dev)
         tl = torch.empty(T, dtype=torch.float32, device=dev)
     nbytes = policy_loss_workspace_bytes(T, H, V)
-    ws = workspace if workspace is not None else _workspace(nbytes, dev, "policy_loss")
+    ws = workspace if workspace is not None else _workspace(nbytes, dev, "policy_loss", stream)
     _check(load().molt_policy_loss_fwd_bwd(
         _bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"), _ptr(tokens, torch.int32, "tokens"),
         _ptr(behavior_logp, torch.float32, "behavior_logp"), _ptr(adv, torch.float32, "adv"),
@@ -434,7 +436,7 @@ def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None
     nbytes = int(load().molt_policy_loss_workspace_bytes_ex(T, H, V, ctypes.byref(opts)))
     if nbytes == 0:
         raise MoltError(2, "unsupported shape for these options")
-    ws = workspace if workspace is not None else _workspace(nbytes, dev, "policy_loss")
+    ws = workspace if workspace is not None else _workspace(nbytes, dev, "policy_loss", stream)
     _check(load().molt_policy_loss_fwd_bwd_ex(
         _bf16_bits(hidden, "hidden"), _bf16_bits(weight, "weight"), _ptr(tokens, torch.int32, "tokens"),
         _ptr(behavior_logp, torch.float32, "behavior_logp"), _ptr(adv, torch.float32, "adv"),

@@ -83,3 +83,31 @@ def test_caller_workspace_and_too_small_workspace():
     with pytest.raises(molt.MoltError):
         molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2, deterministic=True,
                                     workspace=small)
+
+
+def test_concurrent_calls_on_two_streams():
+    """Two different problems issued on two streams at once: each result equals
+    the same problem run alone (the binding gives each stream its workspace)."""
+    probs = []
+    for i in range(2):
+        rng = np.random.default_rng(40 + i)
+        T, H, V = 900, 512, 3000 + 500 * i
+        h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
+        m[0] = 1
+        adv = rng.standard_normal(T).astype(np.float32)
+        b = behavior_from_oracle(O.widen_bf16(h), O.widen_bf16(W), x, 0.3, 0.2, 0.2, 50 + i)
+        probs.append((bf(h), bf(W), t(x), t(b), t(adv), t(m)))
+    alone = [molt.policy_loss_fwd_bwd(*p, 0.2, 0.2) for p in probs]
+    torch.cuda.synchronize()
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    together = []
+    for p, s in zip(probs, streams):
+        with torch.cuda.stream(s):
+            together.append(molt.policy_loss_fwd_bwd(*p, 0.2, 0.2, stream=s))
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    for a, c in zip(alone, together):
+        np.testing.assert_array_equal(np_(a["loss"]), np_(c["loss"]))
+        np.testing.assert_array_equal(np_(a["logp"]), np_(c["logp"]))
+        assert_grad_close(np_(c["dhidden"]), np_(a["dhidden"]).astype(np.float64), "dhidden on a second stream")
+        assert_grad_close(np_(c["dW"]), np_(a["dW"]).astype(np.float64), "dW on a second stream")
