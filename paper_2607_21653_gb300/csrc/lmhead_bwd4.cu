@@ -9,8 +9,8 @@
 // slice of the reduction dimension (vocab for dH, tokens for dW), so every unit
 // drains H-wide fp32 rows into global memory with reduce-adds.  Those drains,
 // together with the operand loads, go through each SM's request path to L2,
-// which moves about 32 B per clock, and that path, not the tensor cores, is what
-// bounds this kernel.  A unit of Tu tokens x Vu vocab drains 4 H (Tu + Vu) bytes
+// which moves about 32 B per clock; with 256 x 256 units that path, not the
+// tensor cores, was the limit.  A unit of Tu tokens x Vu vocab drains 4 H (Tu + Vu) bytes
 // for 6 Tu Vu H flops, so larger units drain less per flop.  The on-chip state
 // that has to grow with the unit is g, which is small (bf16, no H dimension):
 // here a unit is 512 tokens x 512 vocab on four CTAs, twice as deep in both
@@ -48,7 +48,10 @@
 // trip (the MMA frees it, the producer refills it from L2), and the ring's
 // bytes in flight over that latency set the rate at which operands arrive, so
 // the ring is cut fine: a logit stage holds K = 32 of h and W in the 64-byte
-// swizzle, a dH stage 128 vocab rows of W, a dW stage one token tile of h.
+// swizzle, a dH stage 128 vocab rows of W, a dW stage one token tile of h.  With
+// the reduce-adds halved, the 8 MB of operands per unit through this 64 KB ring
+// (all the shared memory GW leaves) and the N = 128 job products are what bound
+// the kernel.
 //
 // Roles per CTA (192 threads): warp 0 TMA producer (each CTA loads its half of
 // every operand; bytes complete on the pair leader's barrier), warp 1 MMA issuer
