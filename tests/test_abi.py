@@ -96,3 +96,21 @@ def test_workspace_query_with_options(lib):
     det = molt.LossOptions(0.0, 0.0, None, None, 0.0, 0.0, 1)
     assert lib.molt_policy_loss_workspace_bytes_ex(1000, 512, 5000, ctypes.byref(det)) >= plain
     assert lib.molt_policy_loss_workspace_bytes_ex(1000, 192, 5000, ctypes.byref(det)) == 0
+
+
+def test_header_compiles_as_c(tmp_path):
+    """include/molt.h is a C header: it compiles with a C11 compiler and -pedantic."""
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "use_header.c"
+    src.write_text('#include "molt.h"\nint main(void) { molt_loss_options o = {0}; (void)o; '
+                   'return (int)(sizeof(molt_stats) + sizeof(molt_stats_ex)); }\n')
+    import os
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([gcc, "-std=c11", "-Wall", "-Wextra", "-pedantic", "-Werror", "-fsyntax-only",
+                        "-I", os.path.join(root, "include"), "-I", "/usr/local/cuda/include", str(src)],
+                       capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
