@@ -465,8 +465,10 @@ def run_ours(args):
     roofline = {
         "kernel": bwd_kernel, "bound": "tensor", "achieved": achieved_bwd, "peak": peak, "unit": "TFLOP/s",
         "frac": achieved_bwd / peak, "traffic": recorded_traffic(bwd_kernel),
-        "limiter": "tensor issue: N=128 pair MMAs take ~1.6x their ideal cycles; operand-stage round trips "
-                   "(~2.5K clocks) with a 64 KB ring",
+        "limiter": ("operand stages: 8 MB per CTA and 512 x 512 unit through a 64 KB ring of 16 KB stages "
+                    "(~3K-clock round trips); the MMA issuer waits for stages ~25% of each unit"
+                    if H % 256 == 0 else
+                    "per-SM reduce-add egress of the fp32 partial products of 128 x 256 units"),
         "peak_source": f"{peaks['source']} bf16 sustained (kernel timed inside a long step)",
         "algorithmic_flops_per_launch": 4.0 * tp * H * V,
         "executed_tflops": 6.0 * tp * H * V / bwd_s / 1e12,

@@ -333,6 +333,9 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   MOLT_TRY(make_tmap(&tm_hz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, 32, kTileM,
                      CU_TENSOR_MAP_SWIZZLE_64B));
   MOLT_TRY(make_tmap(&tm_wz32, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, 32, 128, CU_TENSOR_MAP_SWIZZLE_64B));
+  // 64-row boxes of h: a dW stage of the cluster backward is 64 token rows
+  CUtensorMap tm_h64;
+  MOLT_TRY(make_tmap(&tm_h64, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, 64));
   MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, n_bands * Tcap, H, 32, 32));
   MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
   MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
@@ -379,7 +382,7 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   ba.err = di->status;
   ev_start(3, stream);
   if (pair_bwd)
-    MOLT_CUDA(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
+    MOLT_CUDA(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
               "lmhead backward");
   else
     MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");

@@ -28,34 +28,42 @@
 //          256 columns, the A operand of dH) and into the GW buffers of all four
 //          CTAs: the GW of CTA q holds g of all 512 tokens x vocab quarter q
 //          (MN-major A operand of dW), filled by every CTA for its own tokens.
-//   dH     per 128 columns of H: pair MMA M = 256 tokens, N = 128, K = 512 vocab;
+//   dH     per 256 columns of H: pair MMA M = 256 tokens, N = 256, K = 512 vocab;
 //          A = g from TMEM, B = W rows (MN-major), CTA r staging columns
-//          64 r .. 64 r + 63.
-//   dW     per 128 columns of H: pair MMA M = 256 vocab (the pair's two
-//          quarters), N = 128, K = 512 tokens; A = GW, B = h rows of all four
+//          128 r .. 128 r + 127.
+//   dW     per 256 columns of H: pair MMA M = 256 vocab (the pair's two
+//          quarters), N = 256, K = 512 tokens; A = GW, B = h rows of all four
 //          tiles (MN-major).
 // Partial products drain through swizzled 32 x 32 fp32 boxes with TMA
 // reduce-add into the fp32 dhidden accumulator and dW.
 //
-// TMEM (512 columns per CTA): [0, 256) g; [256, 384) and [384, 512) the job
-// accumulators.  Z_a accumulates over [0, 256) and Z_b over [128, 384); each is
-// converted to g in place (column c of z -> column c / 2 of g), so Z_a of the
-// next unit is computed while the current dW products run, and Z_b once the
-// accumulators are idle.  The epilogue copies each accumulator to registers and
-// hands it back before draining, so one free accumulator keeps the MMAs going.
+// TMEM (512 columns per CTA): [0, 256) g; [256, 512) the job accumulator.  Z_a
+// accumulates over [0, 256) and Z_b over [128, 384); each is converted to g in
+// place (column c of z -> column c / 2 of g), so Z_a of the next unit is
+// computed while the current dW products run, and Z_b once the accumulator is
+// idle.  The job products are N = 256 because a pair MMA of N = 128 takes about
+// 1.6x its ideal clocks and one of N = 256 its ideal 128; that leaves room for a
+// single accumulator, which eight epilogue warps copy to registers (128 columns
+// each) and hand back before draining it.  During the dW products the next
+// unit's Z_a stages fill the MMA issuer's wait for that hand-back.
 //
 // Operands stream through a ring of four 16 KB stages.  Every stage is a round
 // trip (the MMA frees it, the producer refills it from L2), and the ring's
 // bytes in flight over that latency set the rate at which operands arrive, so
 // the ring is cut fine: a logit stage holds K = 32 of h and W in the 64-byte
-// swizzle, a dH stage 128 vocab rows of W, a dW stage one token tile of h.  With
-// the reduce-adds halved, the 8 MB of operands per unit through this 64 KB ring
-// (all the shared memory GW leaves) and the N = 128 job products are what bound
-// the kernel.
+// swizzle, a dH stage 64 vocab rows x 128 columns of W, a dW stage 64 token
+// rows x 128 columns of h.  With the reduce-adds halved and N = 256 job
+// products, the 8 MB of operands per CTA and unit through this 64 KB ring (all
+// the shared memory GW leaves) are what bound the kernel: the MMA issuer waits
+// for operand stages about a quarter of the time.  Neither a fifth stage (paid
+// for with smaller drain boxes) nor multicasting the operands both pairs load
+// made it faster.
 //
-// Roles per CTA (192 threads): warp 0 TMA producer (each CTA loads its half of
+// Roles per CTA (320 threads): warp 0 TMA producer (each CTA loads its half of
 // every operand; bytes complete on the pair leader's barrier), warp 1 MMA issuer
-// (pair leaders only) and TMEM owner, warps 2-5 epilogue.
+// (pair leaders only) and TMEM owner, warps 2-9 epilogue, two per TMEM lane
+// quarter (warp w reads lanes 32 (w % 4) .. 32 (w % 4) + 31, column half
+// (w - 2) / 4).
 #include <atomic>
 #include <cstdint>
 #include <cuda.h>
@@ -75,16 +83,18 @@ constexpr int kOffGW = kStages * kStageBytes;     // 64 KB (1024-aligned)
 constexpr int kGWBlock = 4 * kSub;                // [512 token rows x 64 vocab] bf16, 64 KB
 constexpr int kOffBox = kOffGW + 2 * kGWBlock;    // 192 KB
 constexpr int kBoxBytes = 32 * 32 * 4;
-constexpr int kBoxesPerWarp = 2;
-constexpr int kThreads = 192;
-constexpr int kSmemBytes = 1024 + kOffBox + 4 * kBoxesPerWarp * kBoxBytes;
+constexpr int kEpiWarps = 8;                      // two per TMEM lane quarter
+constexpr int kBoxesPerWarp = 1;
+constexpr int kThreads = 64 + 32 * kEpiWarps;
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr int kSmemBytes = 1024 + kOffBox + kEpiWarps * kBoxesPerWarp * kBoxBytes;
 constexpr uint32_t kIdescZ = idesc_bf16_f32(256, 256, false, false);
-constexpr uint32_t kIdescH = idesc_bf16_f32(256, 128, false, true);   // A from TMEM
-constexpr uint32_t kIdescW = idesc_bf16_f32(256, 128, true, true);
+constexpr uint32_t kIdescH = idesc_bf16_f32(256, 256, false, true);   // A from TMEM
+constexpr uint32_t kIdescW = idesc_bf16_f32(256, 256, true, true);
 constexpr uint32_t kGCol = 0;       // g: 128 tokens x 512 vocab as bf16 pairs
 constexpr uint32_t kZaCol = 0;      // Z of vocab 0..255
 constexpr uint32_t kZbCol = 128;    // Z of vocab 256..511
-constexpr uint32_t kAccCol = 256;   // two 128-column job accumulators
+constexpr uint32_t kAccCol = 256;   // one 256-column job accumulator
 constexpr uint32_t kStageTx = 2u * kStageBytes;   // bytes both CTAs of a pair load per stage
 constexpr float kLog2e = 1.4426950408889634f;
 
@@ -173,8 +183,8 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   __shared__ __align__(8) uint64_t full_bar[kStages];   // pair leader: both CTAs' bytes land here
   __shared__ __align__(8) uint64_t empty_bar[kStages];  // both CTAs of the pair
-  __shared__ __align__(8) uint64_t accf_bar[2];         // both CTAs of the pair: accumulator full
-  __shared__ __align__(8) uint64_t acce_bar[2];         // pair leader: 256 epilogue arrivals
+  __shared__ __align__(8) uint64_t accf_bar;            // both CTAs of the pair: accumulator full
+  __shared__ __align__(8) uint64_t acce_bar;            // pair leader: 512 epilogue arrivals (copied out)
   __shared__ __align__(8) uint64_t zfa_bar;             // every CTA: Z_a done in both pairs (2 commits)
   __shared__ __align__(8) uint64_t zfb_bar;             // every CTA: Z_b done in both pairs (2 commits)
   __shared__ __align__(8) uint64_t ta_bar;              // pair leader: Z_a read, g_a in TMEM (256)
@@ -182,6 +192,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) uint64_t gw_bar;              // pair leader: both GW buffers of the pair full (512)
   __shared__ __align__(8) uint64_t dhd_bar;             // pair leader: this unit's dH products done
   __shared__ __align__(8) uint64_t done_bar;
+  __shared__ __align__(8) uint64_t qsync_bar[4];        // the two epilogue warps of each lane quarter
   __shared__ uint32_t tmem_base_sh;
   __shared__ int abort_sh;
 
@@ -201,17 +212,16 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&full_bar[s]), 1);
       mbar_init(smem_u32(&empty_bar[s]), 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(smem_u32(&accf_bar[b]), 1);
-      mbar_init(smem_u32(&acce_bar[b]), 256);
-    }
+    mbar_init(smem_u32(&accf_bar), 1);
+    mbar_init(smem_u32(&acce_bar), 2 * kEpiThreads);
     mbar_init(smem_u32(&zfa_bar), 2);
     mbar_init(smem_u32(&zfb_bar), 2);
-    mbar_init(smem_u32(&ta_bar), 256);
-    mbar_init(smem_u32(&tb_bar), 256);
-    mbar_init(smem_u32(&gw_bar), 512);
+    mbar_init(smem_u32(&ta_bar), 2 * kEpiThreads);
+    mbar_init(smem_u32(&tb_bar), 2 * kEpiThreads);
+    mbar_init(smem_u32(&gw_bar), 4 * kEpiThreads);
     mbar_init(smem_u32(&dhd_bar), 1);
     mbar_init(smem_u32(&done_bar), 1);
+    for (int i = 0; i < 4; ++i) mbar_init(smem_u32(&qsync_bar[i]), 64);
     abort_sh = 0;
     fence_mbar_init();
   }
@@ -230,7 +240,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   const int n_vp = (a.V + 511) / 512;
   const int H = a.H, V = a.V;
   const int nZ = H / kZK;        // logit stages per vocab half (4 per dW job)
-  const int nJ = H / 128;        // dH jobs = dW jobs per unit
+  const int nJ = H / 256;        // dH jobs = dW jobs per unit
   const int quad = blockIdx.x >> 2, n_quads = gridDim.x >> 2;
 
   // token tile k of unit tq (a missing tile reads tile 0's rows; its g is 0)
@@ -294,25 +304,27 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         // dH jobs: W rows of the unit's 512 vocab, 128 per stage, this CTA's 64
         // of 128 columns
         for (int i = 0; i < nJ && ok; ++i) {
-          const int x = i * 128 + static_cast<int>(prank) * 64;
-          for (int st = 0; st < 4 && ok; ++st) {
+          const int x = i * 256 + static_cast<int>(prank) * 128;
+          for (int st = 0; st < 8 && ok; ++st) {
             uint32_t sa, fb;
             if (!(ok = next_stage(sa, fb))) break;
-            tma_load_2d_pair(sa, &tm_wn, fb, x, v0 + st * 128);
-            tma_load_2d_pair(sa + 8192, &tm_wn, fb, x, v0 + st * 128 + 64);
+            tma_load_2d_pair(sa, &tm_wn, fb, x, v0 + st * 64);
+            tma_load_2d_pair(sa + 8192, &tm_wn, fb, x + 64, v0 + st * 64);
           }
         }
         // dW jobs: h rows of the four tiles, one per stage, this CTA's 64 of 128
         // columns; the next unit's Z_a stages in between
         for (int j = 0; j < nJ && ok; ++j) {
-          const int x = j * 128 + static_cast<int>(prank) * 64;
-          for (int st = 0; st < 4 && ok; ++st) {
+          const int x = j * 256 + static_cast<int>(prank) * 128;
+          for (int st = 0; st < 8 && ok; ++st) {
             uint32_t sa, fb;
             if (!(ok = next_stage(sa, fb))) break;
-            tma_load_2d_pair(sa, &tm_h, fb, x, t4[st]);
+            const int row = t4[st >> 1] + (st & 1) * 64;
+            tma_load_2d_pair(sa, &tm_h, fb, x, row);
+            tma_load_2d_pair(sa + 8192, &tm_h, fb, x + 64, row);
           }
           if (has_next)
-            for (int kb = 4 * j; kb < 4 * j + 4 && ok; ++kb) ok = load_z(kb, n_row0, n_v0);
+            for (int kb = 8 * j; kb < 8 * j + 8 && ok; ++kb) ok = load_z(kb, n_row0, n_v0);
         }
       }
       if (leader) {
@@ -354,10 +366,10 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         if (kb == nZ - 1) umma_commit_pair_mc(bar, 0xF);
         return true;
       };
-      // wait until accumulator `buf` may be written by job index j
+      // wait until the accumulator may be written by job index j (job j - 1
+      // copied out by both CTAs' epilogues)
       auto acc_free = [&](uint32_t j) -> bool {
-        const uint32_t buf = j & 1u, aph = (j >> 1) & 1u;
-        if (!mbar_wait(smem_u32(&acce_bar[buf]), aph ^ 1u, abort_flag, a.err)) return false;
+        if (!mbar_wait(smem_u32(&acce_bar), (j & 1u) ^ 1u, abort_flag, a.err)) return false;
         tc_fence_after();
         return true;
       };
@@ -371,7 +383,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         const bool has_next = nseq.valid();
         // Z_b over [128, 384): Z_a read by both CTAs and both accumulators idle
         if (!(ok = mbar_wait_cluster(smem_u32(&ta_bar), unit_it & 1u, abort_flag, a.err))) break;
-        if (!(ok = acc_free(jj) && acc_free(jj + 1))) break;
+        if (!(ok = acc_free(jj))) break;
         for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb, kZbCol, smem_u32(&zfb_bar));
         if (!ok) break;
         // dH: A = g from TMEM (K = 512 vocab), B = W rows (MN-major)
@@ -379,21 +391,19 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         tc_fence_after();
         for (int i = 0; i < nJ && ok; ++i) {
           if (!(ok = acc_free(jj))) break;
-          const uint32_t buf = jj & 1u;
-          const uint32_t d = tmem_base + kAccCol + buf * 128;
-          for (int st = 0; st < 4 && ok; ++st) {   // 128 vocab rows per stage
+          const uint32_t d = tmem_base + kAccCol;
+          for (int st = 0; st < 8 && ok; ++st) {   // 64 vocab rows x 128 columns per stage
             uint32_t sa;
             if (!(ok = wait_stage(sa))) break;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const int vb = k >> 2, kk = k & 3;
-              const uint64_t bd = sdesc_sw128(sa + vb * 8192 + kk * 2048, 8192, 1024);
-              umma_bf16_pair_ta(d, tmem_base + kGCol + 8u * static_cast<uint32_t>(st * 8 + k), bd, kIdescH,
+            for (int k = 0; k < 4; ++k) {
+              const uint64_t bd = sdesc_sw128(sa + k * 2048, 8192, 1024);
+              umma_bf16_pair_ta(d, tmem_base + kGCol + 8u * static_cast<uint32_t>(st * 4 + k), bd, kIdescH,
                                 (st | k) != 0 ? 1u : 0u);
             }
             release_stage();
           }
-          umma_commit_pair_mc(smem_u32(&accf_bar[buf]), pair_mask);
+          umma_commit_pair_mc(smem_u32(&accf_bar), pair_mask);
           ++jj;
         }
         if (!ok) break;
@@ -404,27 +414,26 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         tc_fence_after();
         for (int j = 0; j < nJ && ok; ++j) {
           if (!(ok = acc_free(jj))) break;
-          const uint32_t buf = jj & 1u;
-          const uint32_t d = tmem_base + kAccCol + buf * 128;
-          for (int st = 0; st < 4 && ok; ++st) {   // one token tile per stage
+          const uint32_t d = tmem_base + kAccCol;
+          for (int st = 0; st < 8 && ok; ++st) {   // 64 token rows x 128 columns per stage
             uint32_t sa;
             if (!(ok = wait_stage(sa))) break;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const uint64_t ad = sdesc_sw128(gw_base + (st * 8 + k) * 2048, kGWBlock, 1024);
-              const uint64_t bd = sdesc_sw128(sa + k * 2048, 16384, 1024);
+            for (int k = 0; k < 4; ++k) {
+              const uint64_t ad = sdesc_sw128(gw_base + (st * 4 + k) * 2048, kGWBlock, 1024);
+              const uint64_t bd = sdesc_sw128(sa + k * 2048, 8192, 1024);
               umma_bf16_pair(d, ad, bd, kIdescW, (st | k) != 0 ? 1u : 0u);
             }
             release_stage();
           }
-          umma_commit_pair_mc(smem_u32(&accf_bar[buf]), pair_mask);
+          umma_commit_pair_mc(smem_u32(&accf_bar), pair_mask);
           ++jj;
           if (has_next && ok) {
             if (j == 0) {   // the dH products have read g: Z_a may overwrite it
               if (!(ok = mbar_wait(smem_u32(&dhd_bar), unit_it & 1u, abort_flag, a.err))) break;
               tc_fence_after();
             }
-            for (int kb = 4 * j; kb < 4 * j + 4 && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
+            for (int kb = 8 * j; kb < 8 * j + 8 && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
           }
         }
         if (ok && !has_next) ok = mbar_wait(smem_u32(&dhd_bar), unit_it & 1u, abort_flag, a.err);
@@ -435,11 +444,22 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
     }
   } else {
     const int q = warp & 3;
+    const int hf = (warp - 2) >> 2;                       // column half of every TMEM read
     const int r_in = q * 32 + lane;                       // own row = TMEM lane
     const uint32_t lane_off = static_cast<uint32_t>(q * 32) << 16;
     const uint32_t box0 = box_base + (warp - 2) * kBoxesPerWarp * kBoxBytes;
-    const uint32_t acce_lead0 = mapa_shared(smem_u32(&acce_bar[0]), lead);
-    const uint32_t acce_lead1 = mapa_shared(smem_u32(&acce_bar[1]), lead);
+    // the two warps that share this lane quarter meet here (bounded wait; the
+    // tcgen05 fences order one warp's TMEM reads before the other's writes)
+    uint32_t qsync_it = 0;
+    auto pair_warps_sync = [&]() -> bool {
+      tc_fence_before();
+      mbar_arrive(smem_u32(&qsync_bar[q]));
+      const bool w = mbar_wait(smem_u32(&qsync_bar[q]), qsync_it & 1u, abort_flag, a.err);
+      ++qsync_it;
+      tc_fence_after();
+      return w;
+    };
+    const uint32_t acce_lead = mapa_shared(smem_u32(&acce_bar), lead);
     const uint32_t ta_lead = mapa_shared(smem_u32(&ta_bar), lead);
     const uint32_t tb_lead = mapa_shared(smem_u32(&tb_bar), lead);
     const uint32_t gw_lead0 = mapa_shared(smem_u32(&gw_bar), 0);
@@ -450,13 +470,12 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
     bool ok = true;
 
     // z (32 columns at zaddr) -> g for vocab columns vc0 .. vc0+31 of the unit:
-    // into TMEM (16 packed columns at gaddr) and into the GW buffer of the
+    // packed into w (stored to TMEM by the caller) and into the GW buffer of the
     // CTA that owns those columns
-    auto convert32 = [&](uint32_t zaddr, uint32_t gaddr, int vc0, float coef, float ecoef, float mu, float lseL,
+    auto convert32 = [&](uint32_t zaddr, uint32_t (&w)[16], int vc0, float coef, float ecoef, float mu, float lseL,
                          int lx, int nvalid, bool live) {
       float v[32];
       tmem_ld32(zaddr, v);
-      uint32_t w[16];
       if (live) {
         const int lxc = lx - vc0;
         const int nv = nvalid - vc0;
@@ -480,7 +499,6 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) w[j] = 0u;
       }
-      tmem_st16(gaddr, w);
       const int owner = vc0 >> 7;                 // vocab quarter -> CTA
       const int cq = vc0 & 127;
       const uint32_t off = static_cast<uint32_t>((cq >> 6) * kGWBlock) + gw_row;
@@ -494,6 +512,21 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         else
           st_shared_cluster_v4(dst + pos, w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
       }
+    };
+    // one logit half (256 columns of z at zcol, vocab vc_base ..): this warp
+    // converts its 128 columns; both warps of the lane quarter read all their z
+    // before either writes g over it (in place: column c -> c / 2)
+    auto convert_half = [&](uint32_t zrow, uint32_t zcol, uint32_t gcol, int vc_base, float coef, float ecoef,
+                            float mu, float lseL, int lx, int nvalid, bool live) -> bool {
+      uint32_t w[4][16];
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        convert32(zrow + zcol + hf * 128 + 32 * c, w[c], vc_base + hf * 128 + 32 * c, coef, ecoef, mu, lseL, lx,
+                  nvalid, live);
+      if (!pair_warps_sync()) return false;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) tmem_st16(zrow + gcol + hf * 64 + 16 * c, w[c]);
+      return true;
     };
     // one [32 x 32] fp32 slab of this warp's rows -> reduce-add into global
     auto drain_slab = [&](const CUtensorMap* map, const float (&v)[32], int x, int y, bool issue) {
@@ -509,22 +542,22 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
     };
     // one job: copy the accumulator to registers, hand it back, then drain it
     auto drain_job = [&](const CUtensorMap* map, int x0, int y, bool issue) -> bool {
-      const uint32_t buf = jj & 1u, aph = (jj >> 1) & 1u;
-      if (!mbar_wait(smem_u32(&accf_bar[buf]), aph, abort_flag, a.err)) return false;
+      if (!mbar_wait(smem_u32(&accf_bar), jj & 1u, abort_flag, a.err)) return false;
       tc_fence_after();
-      const uint32_t taddr = tmem_base + lane_off + kAccCol + buf * 128;
+      const uint32_t taddr = tmem_base + lane_off + kAccCol + hf * 128;
       float v0[32], v1[32], v2[32], v3[32];
       tmem_ld32(taddr, v0);
       tmem_ld32(taddr + 32, v1);
       tmem_ld32(taddr + 64, v2);
       tmem_ld32(taddr + 96, v3);
       tc_fence_before();
-      mbar_arrive_cluster_relaxed(buf ? acce_lead1 : acce_lead0);
+      mbar_arrive_cluster_relaxed(acce_lead);
       ++jj;
-      drain_slab(map, v0, x0, y, issue);
-      drain_slab(map, v1, x0 + 32, y, issue);
-      drain_slab(map, v2, x0 + 64, y, issue);
-      drain_slab(map, v3, x0 + 96, y, issue);
+      const int xh = x0 + hf * 128;
+      drain_slab(map, v0, xh, y, issue);
+      drain_slab(map, v1, xh + 32, y, issue);
+      drain_slab(map, v2, xh + 64, y, issue);
+      drain_slab(map, v3, xh + 96, y, issue);
       return true;
     };
 
@@ -552,9 +585,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       // Z_a -> g of vocab 0..255: TMEM columns [0, 128), GW of CTAs 0 and 1
       if (!(ok = mbar_wait_cluster(smem_u32(&zfa_bar), unit_it & 1u, abort_flag, a.err))) break;
       tc_fence_after();
-#pragma unroll 1
-      for (int c0 = 0; c0 < 256; c0 += 32)
-        convert32(zrow + kZaCol + c0, zrow + kGCol + c0 / 2, c0, coef, ecoef, mu, lseL, lx, nvalid, live);
+      if (!(ok = convert_half(zrow, kZaCol, kGCol, 0, coef, ecoef, mu, lseL, lx, nvalid, live))) break;
       fence_proxy_async_cluster();
       tc_fence_before();
       mbar_arrive_cluster(ta_lead);
@@ -562,10 +593,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       // Z_b -> g of vocab 256..511: TMEM columns [128, 256), GW of CTAs 2 and 3
       if (!(ok = mbar_wait_cluster(smem_u32(&zfb_bar), unit_it & 1u, abort_flag, a.err))) break;
       tc_fence_after();
-#pragma unroll 1
-      for (int c0 = 0; c0 < 256; c0 += 32)
-        convert32(zrow + kZbCol + c0, zrow + kGCol + 128 + c0 / 2, 256 + c0, coef, ecoef, mu, lseL, lx, nvalid,
-                  live);
+      if (!(ok = convert_half(zrow, kZbCol, kGCol + 128, 256, coef, ecoef, mu, lseL, lx, nvalid, live))) break;
       fence_proxy_async_cluster();
       tc_fence_before();
       mbar_arrive_cluster(tb_lead);
@@ -582,11 +610,11 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       // accumulator), 128 columns of H each
       order_drains();
       const int dh_row = own_row0 + q * 32 + seq.band() * a.det_rows;
-      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 128, dh_row, !own_null);
+      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 256, dh_row, !own_null);
       // dW jobs: this CTA's 128 vocab rows (its quarter), 128 columns of H each
       order_drains();
       const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
-      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 128, vrow, vrow < V);
+      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 256, vrow, vrow < V);
       ++unit_it;
     }
     if (lane == 0) bulk_wait_group<0>();
