@@ -70,6 +70,10 @@ const char* molt_status_string(molt_status s);
 /* Text of the last non-OK status returned on the calling thread. */
 const char* molt_last_error(void);
 int molt_version(void);
+/* Process-wide number of CUDA kernels the library has enqueued so far (every
+ * entry point and device; a call that fails part-way counts what it did
+ * enqueue).  For launch accounting in benchmarks and tests. */
+uint64_t molt_kernel_launches(void);
 
 /* Synchronises `stream`, returns the current device's status word in *flags
  * (MOLT_DEV_* bits) and clears it.  Returns the molt_status of the highest

@@ -108,6 +108,7 @@ def load():
         "molt_status_string": (ctypes.c_char_p, [I32]),
         "molt_last_error": (ctypes.c_char_p, []),
         "molt_version": (I32, []),
+        "molt_kernel_launches": (ctypes.c_uint64, []),
         "molt_device_status": (I32, [P, ctypes.POINTER(ctypes.c_uint32)]),
         "molt_group_advantages": (I32, [P, P, I64, D, P, P]),
         "molt_advantages": (I32, [P, P, I64, I32, D, P, P]),
@@ -255,6 +256,11 @@ def device_status(stream=None) -> int:
     if st not in (0, 3, 4, 6, 8):
         _check(st)
     return int(flags.value)
+
+
+def kernel_launches() -> int:
+    """Process-wide number of kernels the library has enqueued so far."""
+    return int(load().molt_kernel_launches())
 
 
 def group_advantages(rewards, group_ids, eps: float = 1e-6, out=None, stream=None):

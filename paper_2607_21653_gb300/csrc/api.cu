@@ -18,6 +18,10 @@
 __device__ unsigned g_molt_status_word;
 
 namespace molt {
+
+std::atomic<unsigned long long> g_kernel_launches{0};
+void note_launches(int n) { g_kernel_launches.fetch_add(static_cast<unsigned long long>(n), std::memory_order_relaxed); }
+
 namespace {
 
 thread_local std::string t_last_error;
@@ -227,10 +231,72 @@ molt_status get_scratch(Scratch& sc, void* ws, size_t ws_bytes, size_t need, cud
   return MOLT_OK;
 }
 
+// Side lanes of the backward.  Clusters of four leave the SMs that cannot hold
+// a whole cluster idle (8 of 152 on a GB300); the single-CTA backward runs there
+// concurrently on a slice of the vocabulary.  One low-priority side stream and a
+// fork/join event pair per (device, caller stream), created on first use and
+// kept for the life of the process; at most kMaxSideLanes of them (further
+// streams run without the split).
+struct SideLane {
+  int dev = -1;
+  cudaStream_t caller = nullptr;
+  cudaStream_t side = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+constexpr int kMaxSideLanes = 64;
+std::mutex g_side_mu;
+SideLane g_side[kMaxSideLanes];
+int g_side_n = 0;
+
+// the side lane of `caller` on the current device, or nullptr (no lane: run
+// the cluster kernel alone)
+const SideLane* side_lane(cudaStream_t caller) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lk(g_side_mu);
+  for (int i = 0; i < g_side_n; ++i)
+    if (g_side[i].dev == dev && g_side[i].caller == caller) return &g_side[i];
+  if (g_side_n == kMaxSideLanes) return nullptr;
+  // no new streams or events while the caller's stream is being captured
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(caller, &cap) != cudaSuccess || cap != cudaStreamCaptureStatusNone) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  SideLane l;
+  l.dev = dev;
+  l.caller = caller;
+  int least = 0, greatest = 0;
+  bool ok = cudaDeviceGetStreamPriorityRange(&least, &greatest) == cudaSuccess &&
+            cudaStreamCreateWithPriority(&l.side, cudaStreamNonBlocking, least) == cudaSuccess;
+  ok = ok && cudaEventCreateWithFlags(&l.fork, cudaEventDisableTiming) == cudaSuccess;
+  ok = ok && cudaEventCreateWithFlags(&l.join, cudaEventDisableTiming) == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    if (l.join) cudaEventDestroy(l.join);
+    if (l.fork) cudaEventDestroy(l.fork);
+    if (l.side) cudaStreamDestroy(l.side);
+    return nullptr;
+  }
+  g_side[g_side_n] = l;
+  return &g_side[g_side_n++];
+}
+
 #define MOLT_CUDA(call, what)                        \
   do {                                               \
     cudaError_t e_ = (call);                         \
     if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+// a kernel launch: as MOLT_CUDA, and counted on success
+#define MOLT_LAUNCH(call, what)                        \
+  do {                                                 \
+    cudaError_t e_ = (call);                           \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+    note_launches(1);                                  \
   } while (0)
 
 #define MOLT_TRY(call)                   \
@@ -246,8 +312,8 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
                         const Workspace& w, const CUtensorMap& tm_h, const CUtensorMap& tm_w, cudaStream_t s) {
   const int64_t Tcap = round_tiles(T);
   ev_start(0, s);
-  MOLT_CUDA(launch_compact(mask, static_cast<int>(T), w, s), "compact");
-  MOLT_CUDA(launch_gather(hidden, tokens, b, adv, static_cast<int>(T), static_cast<int>(Tcap), static_cast<int>(H),
+  MOLT_LAUNCH(launch_compact(mask, static_cast<int>(T), w, s), "compact");
+  MOLT_LAUNCH(launch_gather(hidden, tokens, b, adv, static_cast<int>(T), static_cast<int>(Tcap), static_cast<int>(H),
                           w, di->n_sm, s),
             "gather");
   ev_stop(0, s);
@@ -263,7 +329,7 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
   fa.zx = w.zx;
   fa.err = di->status;
   ev_start(1, s);
-  MOLT_CUDA(launch_lmhead_fwd(tm_h, tm_w, fa, di->n_sm, s), "lmhead forward");
+  MOLT_LAUNCH(launch_lmhead_fwd(tm_h, tm_w, fa, di->n_sm, s), "lmhead forward");
   ev_stop(1, s);
   return MOLT_OK;
 }
@@ -344,18 +410,18 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   if (token_loss_out) MOLT_CUDA(cudaMemsetAsync(token_loss_out, 0, T * sizeof(float), stream), "memset token loss");
   ev_start(2, stream);
   if (opts) {
-    MOLT_CUDA(launch_merge_stats_ex(static_cast<int>(Tcap), static_cast<int>(V), S, w, logp_out, entropy_out,
+    MOLT_LAUNCH(launch_merge_stats_ex(static_cast<int>(Tcap), static_cast<int>(V), S, w, logp_out, entropy_out,
                                     di->status, stream),
               "merge");
-    MOLT_CUDA(launch_seq_gate(static_cast<int>(T), static_cast<int>(Tcap), ex, w, di->status, stream), "gate");
-    MOLT_CUDA(launch_loss_rows_ex(static_cast<int>(Tcap), denom, clip_lo, clip_hi, ex, w, token_loss_out, stream),
+    MOLT_LAUNCH(launch_seq_gate(static_cast<int>(T), static_cast<int>(Tcap), ex, w, di->status, stream), "gate");
+    MOLT_LAUNCH(launch_loss_rows_ex(static_cast<int>(Tcap), denom, clip_lo, clip_hi, ex, w, token_loss_out, stream),
               "loss rows");
   } else {
-    MOLT_CUDA(launch_merge(true, static_cast<int>(Tcap), static_cast<int>(V), S, denom, clip_lo, clip_hi, w,
+    MOLT_LAUNCH(launch_merge(true, static_cast<int>(Tcap), static_cast<int>(V), S, denom, clip_lo, clip_hi, w,
                            logp_out, entropy_out, token_loss_out, di->status, stream),
               "merge");
   }
-  MOLT_CUDA(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, stats_ex_out, di->status, stream),
+  MOLT_LAUNCH(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, stats_ex_out, di->status, stream),
             "finalize");
   ev_stop(2, stream);
   MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(n_bands) * Tcap * H * sizeof(float), stream),
@@ -381,14 +447,47 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   }
   ba.err = di->status;
   ev_start(3, stream);
-  if (pair_bwd)
-    MOLT_CUDA(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
-              "lmhead backward");
-  else
-    MOLT_CUDA(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  if (pair_bwd) {
+    // vocab split with the single-CTA kernel on the SMs no cluster can use
+    // (raster schedule only: the deterministic bands own whole vocab blocks);
+    // per SM that kernel runs at about half the cluster kernel's rate
+    const int clusters = lmhead_bwd_quad_clusters(di->n_sm);
+    const int spare = di->n_sm - 4 * clusters;
+    int64_t Vq = V;
+    const SideLane* lane = nullptr;
+    if (!det && spare > 0 && V >= 64 * 512) {
+      const double share = 0.5 * spare / (0.5 * spare + 4.0 * clusters);
+      const int64_t side_cols = static_cast<int64_t>(share * static_cast<double>(V));
+      if (side_cols >= kBwdBV && (lane = side_lane(stream)) != nullptr) Vq = (V - side_cols) / 512 * 512;
+    }
+    if (Vq < V) {
+      CUtensorMap tm_wz256;
+      MOLT_TRY(make_tmap(&tm_wz256, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kBwdBV));
+      BwdArgs bq = ba;
+      bq.V = static_cast<int>(Vq);   // columns from Vq on count as padding for the cluster kernel
+      BwdArgs bs = ba;
+      bs.vc_begin = static_cast<int>(Vq / kBwdBV);
+      bs.n_vchunks = static_cast<int>((V - Vq + kBwdBV - 1) / kBwdBV);
+      bs.tile_group = 16;
+      // the cluster kernel is enqueued first so that its clusters take their
+      // SMs before the side kernel's CTAs fill the rest
+      MOLT_CUDA(cudaEventRecord(lane->fork, stream), "backward fork");
+      MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, bq, di->n_sm, stream),
+                "lmhead backward");
+      MOLT_CUDA(cudaStreamWaitEvent(lane->side, lane->fork, 0), "backward fork");
+      MOLT_LAUNCH(launch_lmhead_bwd(tm_h, tm_wz256, tm_wn, tm_dh, tm_dw, bs, spare, lane->side),
+                "lmhead backward (side)");
+      MOLT_CUDA(cudaEventRecord(lane->join, lane->side), "backward join");
+      MOLT_CUDA(cudaStreamWaitEvent(stream, lane->join, 0), "backward join");
+    } else {
+      MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
+                "lmhead backward");
+    }
+  } else
+    MOLT_LAUNCH(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
   ev_stop(3, stream);
   ev_start(4, stream);
-  MOLT_CUDA(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), n_bands, Tcap * H, dhidden_out, di->n_sm,
+  MOLT_LAUNCH(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), n_bands, Tcap * H, dhidden_out, di->n_sm,
                            stream),
             "cast dh");
   ev_stop(4, stream);
@@ -441,6 +540,8 @@ const char* molt_last_error(void) { return t_last_error.c_str(); }
 
 int molt_version(void) { return 1; }
 
+uint64_t molt_kernel_launches(void) { return molt::g_kernel_launches.load(std::memory_order_relaxed); }
+
 void molt_set_timing_events(cudaEvent_t* starts, cudaEvent_t* stops, int n) {
   t_ev_start = starts;
   t_ev_stop = stops;
@@ -473,7 +574,7 @@ molt_status molt_group_advantages(const float* rewards, const int32_t* group_ids
   molt_status st;
   const DeviceInfo* di = device_info(&st);
   if (!di) return st;
-  MOLT_CUDA(launch_group_advantages(rewards, group_ids, static_cast<int>(n_resp), eps, adv_out, di->status, stream),
+  MOLT_LAUNCH(launch_group_advantages(rewards, group_ids, static_cast<int>(n_resp), eps, adv_out, di->status, stream),
             "group advantages");
   return MOLT_OK;
 }
@@ -490,7 +591,7 @@ molt_status molt_advantages(const float* rewards, const int32_t* group_ids, int6
   molt_status st;
   const DeviceInfo* di = device_info(&st);
   if (!di) return st;
-  MOLT_CUDA(launch_advantages(rewards, group_ids, static_cast<int>(n_resp), estimator, eps, adv_out, di->status,
+  MOLT_LAUNCH(launch_advantages(rewards, group_ids, static_cast<int>(n_resp), estimator, eps, adv_out, di->status,
                               stream),
             "advantages");
   return MOLT_OK;
@@ -502,7 +603,7 @@ molt_status molt_broadcast_advantages(const float* adv_resp, const int32_t* resp
     return fail(MOLT_ERR_INVALID_ARG, "sizes out of range");
   if (T == 0) return MOLT_OK;
   if (!adv_resp || !resp_of_token || !adv_tok) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
-  MOLT_CUDA(launch_broadcast(adv_resp, resp_of_token, static_cast<int>(n_resp), static_cast<int>(T), adv_tok, stream),
+  MOLT_LAUNCH(launch_broadcast(adv_resp, resp_of_token, static_cast<int>(n_resp), static_cast<int>(T), adv_tok, stream),
             "broadcast");
   return MOLT_OK;
 }
@@ -512,7 +613,7 @@ molt_status molt_mask_count(const uint8_t* mask, int64_t T, int64_t* count_out, 
   if (!count_out || (T > 0 && !mask)) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
   if (T > 0 && !aligned16(mask)) return fail(MOLT_ERR_INVALID_ARG, "mask must be 16-byte aligned");
   if ((reinterpret_cast<uintptr_t>(count_out) & 7u) != 0) return fail(MOLT_ERR_INVALID_ARG, "count_out misaligned");
-  MOLT_CUDA(launch_mask_count(mask, T, count_out, stream), "mask count");
+  MOLT_LAUNCH(launch_mask_count(mask, T, count_out, stream), "mask count");
   return MOLT_OK;
 }
 
@@ -570,7 +671,7 @@ molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, c
   MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
   if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
   ev_start(2, stream);
-  MOLT_CUDA(launch_merge(false, static_cast<int>(Tcap), static_cast<int>(V), S, 0.0, 0.f, 0.f, w, logp_out,
+  MOLT_LAUNCH(launch_merge(false, static_cast<int>(Tcap), static_cast<int>(V), S, 0.0, 0.f, 0.f, w, logp_out,
                          entropy_out, nullptr, di->status, stream),
             "merge");
   ev_stop(2, stream);

@@ -5,7 +5,9 @@
 //   dH_t = sum_v g_tv W_v          dW_v = sum_t g_tv h_t
 //
 // Neither the logits nor g touch global memory.  A work unit is one 128-row
-// tile of active tokens times one 256-column vocab chunk j:
+// tile of active tokens times one 256-column vocab chunk j (chunks counted from
+// vc_begin, so the kernel can take a slice of the vocabulary while the cluster
+// kernel takes the rest):
 //   job Z    z = h_tile W_j^T on the tensor cores (M=128, N=256, K=H) into TMEM;
 //            the epilogue turns it into g (bf16) and stores it in shared memory
 //            in the 128-byte-swizzled K-major layout
@@ -142,7 +144,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
         const Unit un = unit_of(u, n_tiles, n_vc, a.tile_group);
         const int row0 = a.tile_list[un.tile] * kTileM;
-        const int v0 = un.vc * kBwdBV;
+        const int v0 = (a.vc_begin + un.vc) * kBwdBV;
         const int n_kb4 = min(4, (V - v0 + 63) / 64);
         uint32_t sa, fb;
         for (int kb = 0; kb < kblocks && ok; ++kb) {
@@ -195,7 +197,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       };
       for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
         const Unit un = unit_of(u, n_tiles, n_vc, a.tile_group);
-        const int v0 = un.vc * kBwdBV;
+        const int v0 = (a.vc_begin + un.vc) * kBwdBV;
         const int n_kb4 = min(4, (V - v0 + 63) / 64);
         const int n_mh = (V - v0 > 128) ? 2 : 1;
         uint32_t d, sa;
@@ -290,7 +292,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
       const Unit un = unit_of(u, n_tiles, n_vc, a.tile_group);
       const int row0 = a.tile_list[un.tile] * kTileM;
-      const int v0 = un.vc * kBwdBV;
+      const int v0 = (a.vc_begin + un.vc) * kBwdBV;
       const int n_mh = (V - v0 > 128) ? 2 : 1;
       const int row = row0 + r;
       const float coef = a.coef[row];

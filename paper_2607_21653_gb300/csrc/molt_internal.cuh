@@ -64,6 +64,7 @@ struct BwdArgs {
   const int32_t* tile_list;
   int V, H;
   int n_vchunks;
+  int vc_begin;              // single-CTA backward: first 256-column vocab chunk of its range
   int tile_group;            // token tiles per raster group
   const float* ecoef;        // entropy-bonus coefficient per row, or nullptr
   const float* mu;           // sum_v p_v z_v per row (with ecoef)
@@ -120,6 +121,9 @@ cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, 
                               cudaStream_t s);
 // lmhead_bwd4.cu (clusters of two CTA pairs; H % 256 == 0)
 int lmhead_bwd_quad_clusters(int n_sm);   // clusters one launch runs (= deterministic bands)
+// host: count kernels the library enqueued (molt_kernel_launches)
+void note_launches(int n);
+
 cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& tm_wz, const CUtensorMap& tm_h,
                                    const CUtensorMap& tm_w_n, const CUtensorMap& tm_dh, const CUtensorMap& tm_dw,
                                    const BwdArgs& a, int n_sm, cudaStream_t s);

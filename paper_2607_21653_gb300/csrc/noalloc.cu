@@ -161,6 +161,7 @@ extern "C" molt_status molt_token_logprobs_fwd_noalloc(const uint16_t* hidden, c
 
   noalloc_init_kernel<<<static_cast<int>((T + 255) / 256), 256, 0, stream>>>(static_cast<int>(T), counts, zx);
   if ((e = cudaGetLastError()) != cudaSuccess) return noalloc_fail(MOLT_ERR_CUDA, cudaGetErrorString(e));
+  note_launches(1);
   FwdArgs fa{};
   fa.tok_p = tokens;
   fa.counts = counts;
@@ -174,9 +175,11 @@ extern "C" molt_status molt_token_logprobs_fwd_noalloc(const uint16_t* hidden, c
   fa.err = status_word;
   if ((e = launch_lmhead_fwd(tm_h, tm_w, fa, n_sm, stream)) != cudaSuccess)
     return noalloc_fail(MOLT_ERR_CUDA, cudaGetErrorString(e));
+  note_launches(1);
   noalloc_merge_kernel<<<static_cast<int>((T + 127) / 128), 128, 0, stream>>>(
       static_cast<int>(T), static_cast<int>(V), S, static_cast<int>(Tcap), tokens, mask, part, zx, logp_out,
       entropy_out, status_word);
   if ((e = cudaGetLastError()) != cudaSuccess) return noalloc_fail(MOLT_ERR_CUDA, cudaGetErrorString(e));
+  note_launches(1);
   return MOLT_OK;
 }

@@ -62,6 +62,47 @@ def test_random_shapes(i, T, H, V, det):
     assert_grad_close(np_(out["dW"]), ref["dW"], f"dW case {i}")
 
 
+@pytest.mark.parametrize("V", [32768, 40961])
+def test_vocab_split_with_side_kernel(V):
+    """From 64 x 512 vocab columns on, the raster backward splits the vocabulary:
+    the cluster kernel takes the first columns and the single-CTA kernel the
+    rest, concurrently on a side stream over the SMs that no cluster of four can
+    use.  Targets are placed in both slices; the deterministic schedule does not
+    split, so it launches one kernel fewer (on a GB300: 36 clusters, 8 spare SMs)."""
+    T, H = 700, 256
+    rng = np.random.default_rng(V)
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
+    m[:64] = 1
+    x[:32] = rng.integers(V - 700, V, 32)     # in the side kernel's slice
+    x[32:64] = rng.integers(0, 700, 32)       # in the cluster kernel's first block
+    adv = rng.standard_normal(T).astype(np.float32)
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.28, 11)
+    args = (bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28)
+    n0 = molt.kernel_launches()
+    out = molt.policy_loss_fwd_bwd_ex(*args, deterministic=False)
+    n_split = molt.kernel_launches() - n0
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    ref = O.policy_loss(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), m, 0.2, 0.28)
+    ref["_adv"] = adv.astype(np.float64)
+    assert_loss_close(float(out["loss"].item()), ref)
+    assert np.abs(np_(out["logp"]) - ref["logp"]).max() <= LOGP_ATOL
+    assert_grad_close(np_(out["dhidden"]), ref["dH"], f"dhidden V={V}")
+    dW = np_(out["dW"])
+    assert_grad_close(dW, ref["dW"], f"dW V={V}")
+    assert_grad_close(dW[V - 1024:], ref["dW"][V - 1024:], f"dW last columns V={V}")
+    n0 = molt.kernel_launches()
+    det = molt.policy_loss_fwd_bwd_ex(*args, deterministic=True)
+    n_det = molt.kernel_launches() - n0
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    assert_grad_close(np_(det["dW"]), ref["dW"], f"dW deterministic V={V}")
+    assert n_split in (n_det, n_det + 1)
+    if torch.cuda.get_device_properties(0).multi_processor_count == 152:
+        assert n_split == n_det + 1
+
+
 def test_caller_workspace_and_too_small_workspace():
     rng = np.random.default_rng(3)
     T, H, V = 700, 512, 3000
