@@ -52,10 +52,10 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
 
 
-def recorded_traffic(kernel, workload):
-    """DRAM bytes per launch of `kernel` on `workload` from the ncu summaries
-    under profiles/, or None if no summary matches the workload and the
-    current source of the kernel."""
+def recorded_traffic(kernel, workload, schedule):
+    """DRAM bytes per launch of `kernel` on `workload` under `schedule`
+    ("raster" or "deterministic") from the ncu summaries under profiles/, or
+    None if no summary matches them and the current source of the kernel."""
     import glob
     import hashlib
     for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "*.md"))):
@@ -64,7 +64,8 @@ def recorded_traffic(kernel, workload):
                 if not line.startswith("traffic:"):
                     continue
                 kv = dict(tok.split("=", 1) for tok in line.split()[1:] if "=" in tok)
-                if kv.get("kernel") != kernel or kv.get("workload") != workload:
+                if (kv.get("kernel") != kernel or kv.get("workload") != workload
+                        or kv.get("schedule") != schedule):
                     continue
                 src = os.path.join(ROOT, kv.get("source", ""))
                 if not os.path.isfile(src):
@@ -463,7 +464,8 @@ def run_ours(args):
     bwd_kernel = "lmhead_bwd_quad_kernel" if H % 256 == 0 else "lmhead_bwd_kernel"
     roofline = {
         "kernel": bwd_kernel, "bound": "tensor", "achieved": achieved_bwd, "peak": peak, "unit": "TFLOP/s",
-        "frac": achieved_bwd / peak, "traffic": recorded_traffic(bwd_kernel, w.name),
+        "frac": achieved_bwd / peak,
+        "traffic": recorded_traffic(bwd_kernel, w.name, "deterministic" if args.deterministic else "raster"),
         "limiter": ("operand stages: 8 MB per CTA and 512 x 512 unit through a 64 KB ring of 16 KB stages "
                     "(~3K-clock round trips); the MMA issuer waits for stages ~25% of each unit"
                     if H % 256 == 0 else

@@ -205,13 +205,16 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
  *                 0 <= gate_lo <= gate_hi (gate_hi may be +inf)
  *   deterministic 1: dW and dhidden are bitwise reproducible for the same inputs
  *                 on the same device (no paper counterpart).  The backward then
- *                 fixes the order of every partial-sum reduction: each dW row is
- *                 reduced by one warp in a fixed unit order, and each band of
- *                 vocabulary blocks reduces dhidden into its own fp32 copy, which
- *                 a final pass sums in band order.  Needs H % 256 == 0
+ *                 fixes the order of every partial-sum reduction: each of its C
+ *                 clusters (a multiple of 4) owns one slot of every group of
+ *                 four 512-token quads and every (C/4)-th 512-column vocabulary
+ *                 block; each dW element is reduced by one warp, in group order,
+ *                 into the fp32 dW copy of its quad slot (4 copies), each
+ *                 dhidden row, in block order, into one of C/4 fp32 copies, and
+ *                 final passes sum the copies in copy order.  Needs H % 256 == 0
  *                 (MOLT_ERR_UNSUPPORTED_SHAPE otherwise) and the workspace of
- *                 molt_policy_loss_workspace_bytes_ex (one [T, H] fp32 copy per
- *                 band, about 36 bands on a GB300).  0: reduce-adds in
+ *                 molt_policy_loss_workspace_bytes_ex (C/4 [T, H] and four
+ *                 [V, H] fp32 copies: C = 36 on a GB300).  0: reduce-adds in
  *                 arrival order (results agree to fp32 rounding).
  */
 typedef struct {

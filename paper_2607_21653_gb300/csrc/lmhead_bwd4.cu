@@ -115,52 +115,62 @@ __device__ __forceinline__ QuadUnit quad_unit_of(int u, int n_tq, int n_vp, int 
 }
 
 // The units one cluster processes, in order.  Raster schedule: unit u = quad,
-// quad + n_quads, ... of quad_unit_of.  Deterministic schedule (det > 0 bands,
-// one band per cluster index): band b owns vocab blocks b, b + det, ...; for
-// each block it walks every token quad in order, so each dW row is reduced by
-// one warp in a fixed sequence, and the band's dhidden contributions go to its
-// own copy of the accumulator.
+// quad + n_quads, ... of quad_unit_of.  Deterministic schedule (det > 0 = the
+// number of clusters, a multiple of 4): cluster c takes quad slot s = c % 4 of
+// every group of four token quads and the vocab blocks m, m + det / 4, ... with
+// m = c / 4; it walks the groups in order and, inside a group, its blocks in
+// order.  Every dW element then receives its contributions from one cluster in
+// group order (each quad slot drains into its own dW copy), and every dhidden
+// row from one cluster per residue class m in block order (one dhidden copy per
+// class).  At any time the four clusters of a class work on the same vocab
+// block, as in the raster with groups of four quads.
 struct UnitSeq {
   int n_tq, n_vp, n_q, group, det;
-  int u;            // raster position
-  int b, vp, tq;    // band, vocab block, token quad
-  __device__ __forceinline__ void init(int quad, int n_quads, int ntq, int nvp, int grp, int nbands) {
+  int u;                     // raster position
+  int g, b, slot, m, n_m;    // deterministic: group, vocab block, quad slot, class, classes
+  __device__ __forceinline__ void init(int quad, int n_quads, int ntq, int nvp, int grp, int ndet) {
     n_tq = ntq;
     n_vp = nvp;
     n_q = n_quads;
     group = grp;
-    det = nbands;
+    det = ndet;
     u = quad;
-    b = quad;
-    vp = quad;
-    tq = 0;
+    slot = quad & 3;
+    m = quad >> 2;
+    n_m = ndet >> 2;
+    g = 0;
+    b = m;
     settle();
   }
-  __device__ __forceinline__ void settle() {   // skip bands without vocab blocks
+  __device__ __forceinline__ void settle() {   // skip groups without a quad in this slot
     if (det > 0)
-      while (b < det && (vp >= n_vp || n_tq == 0)) {
-        b += n_q;
-        vp = b;
-        tq = 0;
+      while (4 * g < n_tq && (4 * g + slot >= n_tq || b >= n_vp)) {
+        ++g;
+        b = m;
       }
   }
   __device__ __forceinline__ bool valid() const {
-    return det > 0 ? (b < det && vp < n_vp && n_tq > 0) : (u < n_tq * n_vp);
+    return det > 0 ? (4 * g + slot < n_tq && b < n_vp) : (u < n_tq * n_vp);
   }
   __device__ __forceinline__ QuadUnit cur() const {
-    return det > 0 ? QuadUnit{tq, vp} : quad_unit_of(u, n_tq, n_vp, group);
+    return det > 0 ? QuadUnit{4 * g + slot, b} : quad_unit_of(u, n_tq, n_vp, group);
   }
-  __device__ __forceinline__ int band() const { return det > 0 ? b : 0; }
+  __device__ __forceinline__ int dh_copy() const { return det > 0 ? m : 0; }
+  __device__ __forceinline__ int dw_copy() const { return det > 0 ? slot : 0; }
+  // deterministic: the first of this cluster's units in its group (the previous
+  // contributions to its dW rows came from the previous group)
+  __device__ __forceinline__ bool group_start() const { return det > 0 && b == m; }
   __device__ __forceinline__ void advance() {
     if (det == 0) {
       u += n_q;
       return;
     }
-    if (++tq == n_tq) {
-      tq = 0;
-      vp += det;
-      settle();
+    b += n_m;
+    if (b >= n_vp) {
+      ++g;
+      b = m;
     }
+    settle();
   }
 };
 
@@ -600,21 +610,25 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_arrive_cluster(gw_lead1);
       // deterministic schedule: this warp's earlier reduce-adds into the same
       // rows complete before the next ones are issued
-      auto order_drains = [&]() {
-        if (a.det_bands > 0) {
+      auto order_drains = [&](bool needed) {
+        if (needed) {
           if (lane == 0) bulk_wait_group<0>();
           __syncwarp();
         }
       };
-      // dH jobs: this CTA's 128 token rows (in the band's copy of the
-      // accumulator), 128 columns of H each
-      order_drains();
-      const int dh_row = own_row0 + q * 32 + seq.band() * a.det_rows;
+      // dH jobs: this CTA's 128 token rows (in the class's copy of the
+      // accumulator under the deterministic schedule), 256 columns of H each;
+      // the cluster's previous unit drained into the same rows
+      order_drains(a.det_bands > 0);
+      const int dh_row = own_row0 + q * 32 + seq.dh_copy() * a.det_rows;
       for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 256, dh_row, !own_null);
-      // dW jobs: this CTA's 128 vocab rows (its quarter), 128 columns of H each
-      order_drains();
+      // dW jobs: this CTA's 128 vocab rows (its quarter; in the quad slot's
+      // copy under the deterministic schedule), 256 columns of H each; the
+      // previous drains into these rows came from the previous group
+      order_drains(seq.group_start());
       const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
-      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 256, vrow, vrow < V);
+      const int dw_row = vrow + seq.dw_copy() * a.det_vrows;
+      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 256, dw_row, vrow < V);
       ++unit_it;
     }
     if (lane == 0) bulk_wait_group<0>();
@@ -658,6 +672,8 @@ int lmhead_bwd_quad_max_clusters(int n_sm) {
   return n;
 }
 
+int lmhead_bwd_quad_det_clusters(int n_sm) { return lmhead_bwd_quad_clusters(n_sm) / 4 * 4; }
+
 int lmhead_bwd_quad_clusters(int n_sm) {
   int clusters = lmhead_bwd_quad_max_clusters(n_sm);
   if (clusters > n_sm / 4) clusters = n_sm / 4;
@@ -674,8 +690,11 @@ cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& 
                       : cudaFuncSetAttribute(lmhead_bwd_quad_kernel<false>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return e;
-  const int clusters = lmhead_bwd_quad_clusters(n_sm);
-  if (a.det_bands > 0 && a.det_bands != clusters) return cudaErrorInvalidValue;
+  int clusters = lmhead_bwd_quad_clusters(n_sm);
+  if (a.det_bands > 0) {
+    if (a.det_bands > clusters || a.det_bands % 4 != 0) return cudaErrorInvalidValue;
+    clusters = a.det_bands;
+  }
   if (ent)
     lmhead_bwd_quad_kernel<true>
         <<<4 * clusters, kThreads, kSmemBytes, s>>>(tm_hz, tm_wz, tm_h, tm_w_n, tm_dh, tm_dw, a);

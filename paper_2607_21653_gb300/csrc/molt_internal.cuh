@@ -31,7 +31,8 @@ struct Workspace {
   int32_t* tile_flag;   // [Tcap/128]
   int32_t* tile_list;   // [Tcap/128]
   double* red;          // [n_tiles * kRedSlots] per-tile partial sums
-  float* dh32;          // [Tcap, H] fp32 dhidden accumulator (loss call only)
+  float* dh32;          // [copies, Tcap, H] fp32 dhidden accumulator(s) (loss call only)
+  float* dwc;           // [4, V, H] fp32 dW copies of the deterministic schedule, or nullptr
   // extended objective (loss call only)
   float* lp_p;          // [Tcap] packed log-probs
   float* ent_p;         // [Tcap] packed entropies
@@ -70,8 +71,11 @@ struct BwdArgs {
   const float* mu;           // sum_v p_v z_v per row (with ecoef)
   float* dh32;               // [Tcap, H] fp32 dhidden accumulator
   float* dW;                 // [V, H] fp32 dW
-  int det_bands;             // 0: raster schedule; > 0: deterministic bands (one per cluster)
-  int det_rows;              // rows between the bands' dhidden accumulator copies (Tcap)
+  int det_bands;             // 0: raster schedule; > 0: deterministic schedule on this many
+                             // clusters (a multiple of 4): det_bands / 4 dhidden copies and
+                             // 4 dW copies, one per quad slot
+  int det_rows;              // rows between the dhidden accumulator copies (Tcap)
+  int det_vrows;             // rows between the dW copies (V)
   unsigned* err;
 };
 
@@ -115,12 +119,17 @@ cudaError_t launch_loss_rows_ex(int Tcap, double denom, float clip_lo, float cli
 // dhidden_out[t] = bf16(sum over the n_copies accumulator copies, in copy order)
 cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, int n_copies, int64_t copy_stride, uint16_t* dh_out,
                            int n_sm, cudaStream_t s);
+// out = (accumulate ? out : 0) + copies[0] + ... + copies[n_copies - 1], in that
+// order (n elements, a multiple of 4; copies n elements apart)
+cudaError_t launch_sum_copies(const float* copies, int64_t n, int n_copies, float* out, bool accumulate, int n_sm,
+                              cudaStream_t s);
 
 // lmhead_fwd.cu
 cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,
                               cudaStream_t s);
 // lmhead_bwd4.cu (clusters of two CTA pairs; H % 256 == 0)
-int lmhead_bwd_quad_clusters(int n_sm);   // clusters one launch runs (= deterministic bands)
+int lmhead_bwd_quad_clusters(int n_sm);       // clusters one raster launch runs
+int lmhead_bwd_quad_det_clusters(int n_sm);   // clusters of the deterministic schedule (multiple of 4)
 // host: count kernels the library enqueued (molt_kernel_launches)
 void note_launches(int n);
 

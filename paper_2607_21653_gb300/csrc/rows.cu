@@ -594,6 +594,22 @@ __global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __
 
 }  // namespace
 
+// deterministic dW: the quad slots' copies summed in slot order
+__global__ void sum_copies_kernel(const float4* __restrict__ copies, int64_t n4, int n_copies, float4* out,
+                                  int accumulate) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
+    float4 a = accumulate ? out[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = 0; c < n_copies; ++c) {
+      const float4 v = copies[c * n4 + i];
+      a.x += v.x;
+      a.y += v.y;
+      a.z += v.z;
+      a.w += v.w;
+    }
+    out[i] = a;
+  }
+}
+
 cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
                                     unsigned* err, cudaStream_t s) {
   return launch_advantages(rewards, gids, n, kAdvGrpo, eps, out, err, s);
@@ -690,6 +706,14 @@ cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* 
   finalize_kernel<<<1, 1024, 0, s>>>(denom, ws.counts, ws.tile_flag, ws.tile_list, ws.red, loss_out,
                                      reinterpret_cast<StatsDev*>(stats_out),
                                      reinterpret_cast<StatsExDev*>(stats_ex_out), err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_sum_copies(const float* copies, int64_t n, int n_copies, float* out, bool accumulate, int n_sm,
+                              cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  sum_copies_kernel<<<n_sm * 8, 256, 0, s>>>(reinterpret_cast<const float4*>(copies), n / 4, n_copies,
+                                             reinterpret_cast<float4*>(out), accumulate ? 1 : 0);
   return cudaGetLastError();
 }
 

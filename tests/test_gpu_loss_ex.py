@@ -221,7 +221,10 @@ def test_bad_options_rejected():
 
 
 # ----------------------------------------------------------- deterministic mode
-DET_SHAPES = [(1000, 256, 5000), (513, 512, 4133), (640, 768, 2304), (1, 256, 7)]
+# (5000, 256, 9000): about 7 token quads (two groups of four) and 18 vocab
+# blocks (two per residue class on a GB300), so both reduction orders of the
+# schedule have more than one step
+DET_SHAPES = [(1000, 256, 5000), (513, 512, 4133), (640, 768, 2304), (1, 256, 7), (5000, 256, 9000)]
 
 
 @pytest.mark.parametrize("T,H,V", DET_SHAPES)
