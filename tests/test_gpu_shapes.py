@@ -134,6 +134,37 @@ def test_caller_workspace_and_too_small_workspace():
                                     workspace=small)
 
 
+def test_policy_loss_captured_in_a_cuda_graph():
+    """The loss call captured into a CUDA graph and replayed gives the eager
+    call's results.  The eager call runs first on the same stream, so the
+    stream's workspace and side stream exist and the vocab split (V >= 32768)
+    forks onto the side stream and joins back inside the captured graph."""
+    T, H, V = 700, 256, 40961
+    rng = np.random.default_rng(77)
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    b = behavior_from_oracle(O.widen_bf16(h), O.widen_bf16(W), x, 0.3, 0.2, 0.28, 78)
+    args = (bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        eager = molt.policy_loss_fwd_bwd(*args, stream=s)
+    s.synchronize()
+    assert molt.device_status() == 0
+    eager = {k: v.clone() for k, v in eager.items() if v is not None}
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        out = molt.policy_loss_fwd_bwd(*args, stream=s)
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        assert molt.device_status() == 0
+        np.testing.assert_array_equal(np_(out["loss"]), np_(eager["loss"]))
+        np.testing.assert_array_equal(np_(out["logp"]), np_(eager["logp"]))
+        assert_grad_close(np_(out["dhidden"]), np_(eager["dhidden"]).astype(np.float64), "dhidden (graph replay)")
+        assert_grad_close(np_(out["dW"]), np_(eager["dW"]).astype(np.float64), "dW (graph replay)")
+
+
 def test_concurrent_calls_on_two_streams():
     """Two different problems issued on two streams at once: each result equals
     the same problem run alone (the binding gives each stream its workspace)."""
