@@ -463,8 +463,9 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   ev_start(3, stream);
   if (pair_bwd) {
     // vocab split with the single-CTA kernel on the SMs no cluster can use
-    // (raster schedule only: the deterministic bands own whole vocab blocks);
-    // per SM that kernel runs at about half the cluster kernel's rate
+    // (raster schedule only: the deterministic order needs every vocab block
+    // reduced by its owner clusters); per SM that kernel runs at about half
+    // the cluster kernel's rate
     const int clusters = lmhead_bwd_quad_clusters(di->n_sm);
     const int spare = di->n_sm - 4 * clusters;
     int64_t Vq = V;
@@ -489,10 +490,14 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
       MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, bq, di->n_sm, stream),
                 "lmhead backward");
       MOLT_CUDA(cudaStreamWaitEvent(lane->side, lane->fork, 0), "backward fork");
-      MOLT_LAUNCH(launch_lmhead_bwd(tm_h, tm_wz256, tm_wn, tm_dh, tm_dw, bs, spare, lane->side),
-                "lmhead backward (side)");
-      MOLT_CUDA(cudaEventRecord(lane->join, lane->side), "backward join");
-      MOLT_CUDA(cudaStreamWaitEvent(stream, lane->join, 0), "backward join");
+      // the join is made whatever the side launch returned, so that nothing on
+      // the caller's stream (the workspace release included) can overtake it
+      const cudaError_t e_side = launch_lmhead_bwd(tm_h, tm_wz256, tm_wn, tm_dh, tm_dw, bs, spare, lane->side);
+      if (e_side == cudaSuccess) note_launches(1);
+      cudaError_t e_join = cudaEventRecord(lane->join, lane->side);
+      if (e_join == cudaSuccess) e_join = cudaStreamWaitEvent(stream, lane->join, 0);
+      if (e_side != cudaSuccess) return cuda_fail(e_side, "lmhead backward (side)");
+      if (e_join != cudaSuccess) return cuda_fail(e_join, "backward join");
     } else {
       MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
                 "lmhead backward");
