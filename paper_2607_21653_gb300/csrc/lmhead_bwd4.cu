@@ -38,10 +38,11 @@
 // reduce-add into the fp32 dhidden accumulator and dW.
 //
 // TMEM (512 columns per CTA): [0, 256) g; [256, 512) the job accumulator.  Z_a
-// accumulates over [0, 256) and Z_b over [128, 384); each is converted to g in
-// place (column c of z -> column c / 2 of g), so Z_a of the next unit is
-// computed while the current dW products run, and Z_b once the accumulator is
-// idle.  The job products are N = 256 because a pair MMA of N = 128 takes about
+// accumulates over [0, 256) and is converted to g in place (column c of z ->
+// column c / 2 of g), so Z_a of the next unit is computed while the current dW
+// products run; Z_b accumulates over the accumulator's columns once they are
+// idle and is converted into g columns [128, 256) after Z_a's conversion has
+// read them.  The job products are N = 256 because a pair MMA of N = 128 takes about
 // 1.6x its ideal clocks and one of N = 256 its ideal 128; that leaves room for a
 // single accumulator, which eight epilogue warps copy to registers (128 columns
 // each) and hand back before draining it.  During the dW products the next
@@ -93,7 +94,7 @@ constexpr uint32_t kIdescH = idesc_bf16_f32(256, 256, false, true);   // A from 
 constexpr uint32_t kIdescW = idesc_bf16_f32(256, 256, true, true);
 constexpr uint32_t kGCol = 0;       // g: 128 tokens x 512 vocab as bf16 pairs
 constexpr uint32_t kZaCol = 0;      // Z of vocab 0..255
-constexpr uint32_t kZbCol = 128;    // Z of vocab 256..511
+constexpr uint32_t kZbCol = 256;    // Z of vocab 256..511 (over the idle accumulator)
 constexpr uint32_t kAccCol = 256;   // one 256-column job accumulator
 constexpr uint32_t kStageTx = 2u * kStageBytes;   // bytes both CTAs of a pair load per stage
 constexpr float kLog2e = 1.4426950408889634f;
@@ -197,7 +198,6 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) uint64_t acce_bar;            // pair leader: 512 epilogue arrivals (copied out)
   __shared__ __align__(8) uint64_t zfa_bar;             // every CTA: Z_a done in both pairs (2 commits)
   __shared__ __align__(8) uint64_t zfb_bar;             // every CTA: Z_b done in both pairs (2 commits)
-  __shared__ __align__(8) uint64_t ta_bar;              // pair leader: Z_a read, g_a in TMEM (256)
   __shared__ __align__(8) uint64_t tb_bar;              // pair leader: Z_b read, g_b in TMEM (256)
   __shared__ __align__(8) uint64_t gw_bar;              // pair leader: both GW buffers of the pair full (512)
   __shared__ __align__(8) uint64_t dhd_bar;             // pair leader: this unit's dH products done
@@ -226,7 +226,6 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
     mbar_init(smem_u32(&acce_bar), 2 * kEpiThreads);
     mbar_init(smem_u32(&zfa_bar), 2);
     mbar_init(smem_u32(&zfb_bar), 2);
-    mbar_init(smem_u32(&ta_bar), 2 * kEpiThreads);
     mbar_init(smem_u32(&tb_bar), 2 * kEpiThreads);
     mbar_init(smem_u32(&gw_bar), 4 * kEpiThreads);
     mbar_init(smem_u32(&dhd_bar), 1);
@@ -391,8 +390,8 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         UnitSeq nseq = seq;
         nseq.advance();
         const bool has_next = nseq.valid();
-        // Z_b over [128, 384): Z_a read by both CTAs and both accumulators idle
-        if (!(ok = mbar_wait_cluster(smem_u32(&ta_bar), unit_it & 1u, abort_flag, a.err))) break;
+        // Z_b over [256, 512) once the accumulator is idle (its conversion
+        // writes g columns [128, 256) after Z_a's has read them)
         if (!(ok = acc_free(jj))) break;
         for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb, kZbCol, smem_u32(&zfb_bar));
         if (!ok) break;
@@ -470,7 +469,6 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       return w;
     };
     const uint32_t acce_lead = mapa_shared(smem_u32(&acce_bar), lead);
-    const uint32_t ta_lead = mapa_shared(smem_u32(&ta_bar), lead);
     const uint32_t tb_lead = mapa_shared(smem_u32(&tb_bar), lead);
     const uint32_t gw_lead0 = mapa_shared(smem_u32(&gw_bar), 0);
     const uint32_t gw_lead1 = mapa_shared(smem_u32(&gw_bar), 2);
@@ -598,7 +596,6 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       if (!(ok = convert_half(zrow, kZaCol, kGCol, 0, coef, ecoef, mu, lseL, lx, nvalid, live))) break;
       fence_proxy_async_cluster();
       tc_fence_before();
-      mbar_arrive_cluster(ta_lead);
       mbar_arrive_cluster(gw_lead0);
       // Z_b -> g of vocab 256..511: TMEM columns [128, 256), GW of CTAs 2 and 3
       if (!(ok = mbar_wait_cluster(smem_u32(&zfb_bar), unit_it & 1u, abort_flag, a.err))) break;
