@@ -52,12 +52,25 @@ def load_peaks():
     return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
 
 
+def code_hash(path):
+    """First 16 hex digits of the sha256 of a C++/CUDA source with its comments
+    removed and its whitespace collapsed: edits to comments leave it unchanged,
+    any change to the code does not."""
+    import hashlib
+    import re
+    with open(path, encoding="utf-8") as f:
+        src = f.read()
+    src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", " ", src)
+    src = " ".join(src.split())
+    return hashlib.sha256(src.encode()).hexdigest()[:16]
+
+
 def recorded_traffic(kernel, workload, schedule):
     """DRAM bytes per launch of `kernel` on `workload` under `schedule`
     ("raster" or "deterministic") from the ncu summaries under profiles/, or
     None if no summary matches them and the current source of the kernel."""
     import glob
-    import hashlib
     for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "*.md"))):
         with open(path) as f:
             for line in f:
@@ -68,11 +81,7 @@ def recorded_traffic(kernel, workload, schedule):
                         or kv.get("schedule") != schedule):
                     continue
                 src = os.path.join(ROOT, kv.get("source", ""))
-                if not os.path.isfile(src):
-                    continue
-                with open(src, "rb") as fs:
-                    digest = hashlib.sha256(fs.read()).hexdigest()[:16]
-                if digest == kv.get("sha256_16"):
+                if os.path.isfile(src) and code_hash(src) == kv.get("code_sha256_16"):
                     return float(kv["dram_bytes_per_launch"])
     return None
 

@@ -198,8 +198,8 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) uint64_t acce_bar;            // pair leader: 512 epilogue arrivals (copied out)
   __shared__ __align__(8) uint64_t zfa_bar;             // every CTA: Z_a done in both pairs (2 commits)
   __shared__ __align__(8) uint64_t zfb_bar;             // every CTA: Z_b done in both pairs (2 commits)
-  __shared__ __align__(8) uint64_t tb_bar;              // pair leader: Z_b read, g_b in TMEM (256)
-  __shared__ __align__(8) uint64_t gw_bar;              // pair leader: both GW buffers of the pair full (512)
+  __shared__ __align__(8) uint64_t tb_bar;              // pair leader: Z_b read, g_b in TMEM (both CTAs' epilogues)
+  __shared__ __align__(8) uint64_t gw_bar;              // pair leader: both GW buffers of the pair full (all 4 CTAs)
   __shared__ __align__(8) uint64_t dhd_bar;             // pair leader: this unit's dH products done
   __shared__ __align__(8) uint64_t done_bar;
   __shared__ __align__(8) uint64_t qsync_bar[4];        // the two epilogue warps of each lane quarter
