@@ -93,6 +93,13 @@ def test_vocab_split_with_side_kernel(V):
     dW = np_(out["dW"])
     assert_grad_close(dW, ref["dW"], f"dW V={V}")
     assert_grad_close(dW[V - 1024:], ref["dW"][V - 1024:], f"dW last columns V={V}")
+    # accumulating into a caller's dW: both kernels add onto it
+    dW0 = torch.randn(V, H, device="cuda", generator=torch.Generator(device="cuda").manual_seed(V))
+    acc = dW0.clone()
+    molt.policy_loss_fwd_bwd_ex(*args, deterministic=False, dW=acc, accumulate_dW=True)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    assert_grad_close(np_(acc - dW0), ref["dW"], f"dW accumulated V={V}")
     det = molt.policy_loss_fwd_bwd_ex(*args, deterministic=True)
     torch.cuda.synchronize()
     assert molt.device_status() == 0
