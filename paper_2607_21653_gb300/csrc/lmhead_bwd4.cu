@@ -310,8 +310,8 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         }
         // Z_b of this unit
         for (int kb = 0; kb < nZ && ok; ++kb) ok = load_z(kb, own_row0, v0 + 256);
-        // dH jobs: W rows of the unit's 512 vocab, 128 per stage, this CTA's 64
-        // of 128 columns
+        // dH jobs: W rows of the unit's 512 vocab, 64 per stage, this CTA's 128
+        // of the job's 256 columns
         for (int i = 0; i < nJ && ok; ++i) {
           const int x = i * 256 + static_cast<int>(prank) * 128;
           for (int st = 0; st < 8 && ok; ++st) {
@@ -321,8 +321,8 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
             tma_load_2d_pair(sa + 8192, &tm_wn, fb, x + 64, v0 + st * 64);
           }
         }
-        // dW jobs: h rows of the four tiles, one per stage, this CTA's 64 of 128
-        // columns; the next unit's Z_a stages in between
+        // dW jobs: h rows of the four tiles, 64 per stage, this CTA's 128 of the
+        // job's 256 columns; the next unit's Z_a stages in between
         for (int j = 0; j < nJ && ok; ++j) {
           const int x = j * 256 + static_cast<int>(prank) * 128;
           for (int st = 0; st < 8 && ok; ++st) {
