@@ -215,6 +215,34 @@ struct Scratch {
   }
 };
 
+// Vocab split of the raster backward (see the side lanes below): the first
+// Vq columns go to the cluster kernel, the rest to the single-CTA kernel on the
+// `spare` SMs.  Vq is the multiple of 512 that minimises the later of the two
+// kernels' predicted finish times, in units per cluster (512 x 512 units over
+// `clusters`) against units per spare SM (128 x 256 units, measured at 0.84 of
+// a cluster unit's time); T stands in for the active rows.  Returns V for no
+// split.
+int64_t choose_vocab_split(int64_t T, int64_t V, int clusters, int spare) {
+  if (spare <= 0 || clusters <= 0 || V < 16 * 512) return V;
+  const int64_t n_t = (T + kTileM - 1) / kTileM, n_tq = (n_t + 3) / 4;
+  auto cdiv = [](int64_t a, int64_t b) { return (a + b - 1) / b; };
+  auto finish = [&](int64_t vq) {
+    const double quad = static_cast<double>(cdiv(cdiv(vq, 512) * n_tq, clusters));
+    const double side = vq < V ? 0.84 * static_cast<double>(cdiv(cdiv(V - vq, kBwdBV) * n_t, spare)) : 0.0;
+    return quad > side ? quad : side;
+  };
+  int64_t best = V;
+  double best_t = finish(V) * 0.995;   // a split must gain at least 0.5 %
+  for (int64_t vq = (V - 1) / 512 * 512; vq >= V - V / 8 && vq > 0; vq -= 512) {
+    const double t = finish(vq);
+    if (t < best_t) {
+      best_t = t;
+      best = vq;
+    }
+  }
+  return best;
+}
+
 molt_status get_scratch(Scratch& sc, void* ws, size_t ws_bytes, size_t need, cudaStream_t s) {
   sc.s = s;
   if (ws) {
@@ -464,16 +492,14 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   if (pair_bwd) {
     // vocab split with the single-CTA kernel on the SMs no cluster can use
     // (raster schedule only: the deterministic order needs every vocab block
-    // reduced by its owner clusters); per SM that kernel runs at about half
-    // the cluster kernel's rate
+    // reduced by its owner clusters)
     const int clusters = lmhead_bwd_quad_clusters(di->n_sm);
     const int spare = di->n_sm - 4 * clusters;
     int64_t Vq = V;
     const SideLane* lane = nullptr;
-    if (!det && spare > 0 && V >= 64 * 512) {
-      const double share = 0.5 * spare / (0.5 * spare + 4.0 * clusters);
-      const int64_t side_cols = static_cast<int64_t>(share * static_cast<double>(V));
-      if (side_cols >= kBwdBV && (lane = side_lane(stream)) != nullptr) Vq = (V - side_cols) / 512 * 512;
+    if (!det) {
+      const int64_t vq = choose_vocab_split(T, V, clusters, spare);
+      if (vq < V && (lane = side_lane(stream)) != nullptr) Vq = vq;
     }
     if (Vq < V) {
       CUtensorMap tm_wz256;

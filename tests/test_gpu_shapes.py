@@ -62,19 +62,21 @@ def test_random_shapes(i, T, H, V, det):
     assert_grad_close(np_(out["dW"]), ref["dW"], f"dW case {i}")
 
 
-@pytest.mark.parametrize("V", [32768, 40961])
+@pytest.mark.parametrize("V", [18986, 19243])
 def test_vocab_split_with_side_kernel(V):
-    """From 64 x 512 vocab columns on, the raster backward splits the vocabulary:
-    the cluster kernel takes the first columns and the single-CTA kernel the
-    rest, concurrently on a side stream over the SMs that no cluster of four can
-    use.  Targets are placed in both slices; the deterministic schedule does not
-    split.  Below the threshold the call launches one kernel fewer (on a GB300:
-    36 clusters, 8 spare SMs)."""
+    """The raster backward splits the vocabulary when that evens out the work:
+    the cluster kernel takes the first whole 512-column blocks and the
+    single-CTA kernel the rest, concurrently on a side stream over the SMs that
+    no cluster of four can use.  With 700 tokens and these V (on a GB300: 36
+    clusters, 8 spare SMs) the cluster kernel keeps 36 blocks and the side
+    kernel takes the last 554 or 811 columns.  Targets are placed in both
+    slices; the deterministic schedule does not split; with V = 18432 (whole
+    blocks, nothing to even out) the call launches one kernel fewer."""
     T, H = 700, 256
     rng = np.random.default_rng(V)
     h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
     m[:64] = 1
-    x[:32] = rng.integers(V - 700, V, 32)     # in the side kernel's slice
+    x[:32] = rng.integers(V - 500, V, 32)     # in the side kernel's slice
     x[32:64] = rng.integers(0, 700, 32)       # in the cluster kernel's first block
     adv = rng.standard_normal(T).astype(np.float32)
     h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
@@ -104,10 +106,9 @@ def test_vocab_split_with_side_kernel(V):
     torch.cuda.synchronize()
     assert molt.device_status() == 0
     assert_grad_close(np_(det["dW"]), ref["dW"], f"dW deterministic V={V}")
-    # one vocab column fewer than the split threshold: the same kernels but the
-    # side one
-    hs, Ws = h, W[: 64 * 512 - 1]
-    xs = np.minimum(x, 64 * 512 - 2).astype(x.dtype)
+    # 36 whole blocks: the same kernels but the side one
+    hs, Ws = h, W[:18432]
+    xs = np.minimum(x, 18431).astype(x.dtype)
     n0 = molt.kernel_launches()
     molt.policy_loss_fwd_bwd_ex(bf(hs), bf(Ws), t(xs), t(b), t(adv), t(m), 0.2, 0.28, deterministic=False)
     n_plain = molt.kernel_launches() - n0
@@ -144,9 +145,10 @@ def test_caller_workspace_and_too_small_workspace():
 def test_policy_loss_captured_in_a_cuda_graph():
     """The loss call captured into a CUDA graph and replayed gives the eager
     call's results.  The eager call runs first on the same stream, so the
-    stream's workspace and side stream exist and the vocab split (V >= 32768)
-    forks onto the side stream and joins back inside the captured graph."""
-    T, H, V = 700, 256, 40961
+    stream's workspace and side stream exist and the vocab split (chosen for
+    700 tokens and V = 18986 on a GB300) forks onto the side stream and joins
+    back inside the captured graph."""
+    T, H, V = 700, 256, 18986
     rng = np.random.default_rng(77)
     h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
     m[0] = 1
