@@ -37,6 +37,15 @@ def test_rejects_unsupported_hidden(lib):
     assert "multiple of 64" in lib.molt_last_error().decode()
 
 
+def test_launch_counter_unchanged_by_rejected_calls(lib):
+    """molt_kernel_launches counts kernels actually enqueued: a call that
+    fails validation enqueues none."""
+    n0 = lib.molt_kernel_launches()
+    st = lib.molt_token_logprobs_fwd(FAKE, FAKE, FAKE, None, 16, 100, 32, FAKE, None, None, 0, None)
+    assert molt.STATUS[st] == "MOLT_ERR_UNSUPPORTED_SHAPE"
+    assert lib.molt_kernel_launches() == n0
+
+
 def test_rejects_null_and_misaligned(lib):
     st = lib.molt_token_logprobs_fwd(None, FAKE, FAKE, None, 16, 64, 32, FAKE, None, None, 0, None)
     assert molt.STATUS[st] == "MOLT_ERR_INVALID_ARG"
