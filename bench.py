@@ -470,20 +470,20 @@ def run_ours(args):
     achieved_bwd = 4.0 * tp * H * V / bwd_s / 1e12
     step_s = ms / 1e3 / args.steps
     step_frac = 6.0 * tp * H * V / step_s / 1e12 / peak
-    bwd_kernel = "lmhead_bwd_quad_kernel" if H % 256 == 0 else "lmhead_bwd_kernel"
+    bwd_kernel = "lmhead_bwd_quad_kernel" if H % 128 == 0 else "lmhead_bwd_kernel"
     roofline = {
         "kernel": bwd_kernel, "bound": "tensor", "achieved": achieved_bwd, "peak": peak, "unit": "TFLOP/s",
         "frac": achieved_bwd / peak,
         "traffic": recorded_traffic(bwd_kernel, w.name, "deterministic" if args.deterministic else "raster"),
         "limiter": ("operand stages: 8 MB per CTA and 512 x 512 unit through a 64 KB ring of 16 KB stages "
                     "(~3K-clock round trips); the MMA issuer waits for stages ~25% of each unit"
-                    if H % 256 == 0 else
+                    if H % 128 == 0 else
                     "per-SM reduce-add egress of the fp32 partial products of 128 x 256 units"),
         "peak_source": f"{peaks['source']} bf16 sustained (kernel timed inside a long step)",
         "concurrent": ("when the call splits the vocabulary (raster schedule; the library picks the split "
                        "that evens out the two kernels), lmhead_bwd_kernel runs on the SMs no cluster of four "
                        "can use over the last few percent of it; achieved and the event time cover both"
-                       if H % 256 == 0 and not args.deterministic else None),
+                       if H % 128 == 0 and not args.deterministic else None),
         "kernels_per_step": launches / args.steps,
         "algorithmic_flops_per_launch": 4.0 * tp * H * V,
         "executed_tflops": 6.0 * tp * H * V / bwd_s / 1e12,

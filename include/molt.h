@@ -211,7 +211,7 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
  *                 block; each dW element is reduced by one warp, in group order,
  *                 into the fp32 dW copy of its quad slot (4 copies), each
  *                 dhidden row, in block order, into one of C/4 fp32 copies, and
- *                 final passes sum the copies in copy order.  Needs H % 256 == 0
+ *                 final passes sum the copies in copy order.  Needs H % 128 == 0
  *                 (MOLT_ERR_UNSUPPORTED_SHAPE otherwise) and the workspace of
  *                 molt_policy_loss_workspace_bytes_ex (C/4 [T, H] and four
  *                 [V, H] fp32 copies: C = 36 on a GB300).  0: reduce-adds in

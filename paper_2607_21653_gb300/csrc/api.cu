@@ -400,7 +400,7 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
       return fail(MOLT_ERR_INVALID_ARG, "the gate band must satisfy 0 <= gate_lo <= gate_hi");
   }
   const bool det = opts && opts->deterministic;
-  if (det && H % 256 != 0) return fail(MOLT_ERR_UNSUPPORTED_SHAPE, "deterministic mode needs H % 256 == 0");
+  if (det && H % 128 != 0) return fail(MOLT_ERR_UNSUPPORTED_SHAPE, "deterministic mode needs H % 128 == 0");
   molt_status st;
   const DeviceInfo* di = device_info(&st);
   if (!di) return st;
@@ -423,7 +423,7 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   Scratch sc;
   MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
   const Workspace w = carve(sc.ptr, L);
-  const bool pair_bwd = (H % 256) == 0;
+  const bool pair_bwd = (H % 128) == 0;   // the cluster backward
   CUtensorMap tm_h, tm_w, tm_wz, tm_wn, tm_dh, tm_dw;
   MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
   MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
@@ -685,7 +685,7 @@ size_t molt_policy_loss_workspace_bytes(int64_t T, int64_t H, int64_t V) {
 size_t molt_policy_loss_workspace_bytes_ex(int64_t T, int64_t H, int64_t V, const molt_loss_options* opts) {
   if (check_shape(T, H, V) != MOLT_OK) return 0;
   const bool det = opts && opts->deterministic;
-  if (det && H % 256 != 0) return 0;
+  if (det && H % 128 != 0) return 0;
   molt_status st;
   const DeviceInfo* di = device_info(&st);
   const int n_sm = di ? di->n_sm : 152;

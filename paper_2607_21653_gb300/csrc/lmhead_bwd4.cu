@@ -1,5 +1,5 @@
 // Backward pass of the fused LM-head + policy loss on clusters of four CTAs
-// (two tcgen05 CTA pairs), used when H is a multiple of 256.
+// (two tcgen05 CTA pairs), used when H is a multiple of 128.
 //
 //   g_tv = coef_t (softmax(z_t)_v - [v == x_t]),  coef_t = m_t c_t / D   (Eq. 2)
 //          (+ ecoef_t softmax(z_t)_v (z_tv - mu_t) with an entropy bonus)
@@ -92,6 +92,8 @@ constexpr int kSmemBytes = 1024 + kOffBox + kEpiWarps * kBoxesPerWarp * kBoxByte
 constexpr uint32_t kIdescZ = idesc_bf16_f32(256, 256, false, false);
 constexpr uint32_t kIdescH = idesc_bf16_f32(256, 256, false, true);   // A from TMEM
 constexpr uint32_t kIdescW = idesc_bf16_f32(256, 256, true, true);
+constexpr uint32_t kIdescH128 = idesc_bf16_f32(256, 128, false, true);   // the last job when H % 256 == 128
+constexpr uint32_t kIdescW128 = idesc_bf16_f32(256, 128, true, true);
 constexpr uint32_t kGCol = 0;       // g: 128 tokens x 512 vocab as bf16 pairs
 constexpr uint32_t kZaCol = 0;      // Z of vocab 0..255
 constexpr uint32_t kZbCol = 256;    // Z of vocab 256..511 (over the idle accumulator)
@@ -249,7 +251,9 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   const int n_vp = (a.V + 511) / 512;
   const int H = a.H, V = a.V;
   const int nZ = H / kZK;        // logit stages per vocab half (4 per dW job)
-  const int nJ = H / 256;        // dH jobs = dW jobs per unit
+  const int nJ = (H + 255) / 256;   // dH jobs = dW jobs per unit
+  // columns of H job j covers: 256, except a last job of 128 when H % 256 == 128
+  auto job_w = [&](int j) -> int { return (H & 255) != 0 && j == nJ - 1 ? 128 : 256; };
   const int quad = blockIdx.x >> 2, n_quads = gridDim.x >> 2;
 
   // token tile k of unit tq (a missing tile reads tile 0's rows; its g is 0)
@@ -268,12 +272,12 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       for (int s = 0; s < kStages; ++s) full_leader[s] = mapa_shared(smem_u32(&full_bar[s]), lead);
       uint32_t it = 0;
       bool ok = true;
-      auto next_stage = [&](uint32_t& sa, uint32_t& fb) -> bool {
+      auto next_stage = [&](uint32_t& sa, uint32_t& fb, uint32_t tx = kStageTx) -> bool {
         const uint32_t st = it % kStages, ph = (it / kStages) & 1u;
         if (!mbar_wait(smem_u32(&empty_bar[st]), ph ^ 1u, abort_flag, a.err)) return false;
         sa = smem0 + st * kStageBytes;
         fb = full_leader[st];
-        if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[st]), kStageTx);
+        if (leader) mbar_arrive_expect_tx(smem_u32(&full_bar[st]), tx);
         ++it;
         return true;
       };
@@ -313,27 +317,29 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         // dH jobs: W rows of the unit's 512 vocab, 64 per stage, this CTA's 128
         // of the job's 256 columns
         for (int i = 0; i < nJ && ok; ++i) {
-          const int x = i * 256 + static_cast<int>(prank) * 128;
+          const int w = job_w(i);
+          const int x = i * 256 + static_cast<int>(prank) * (w / 2);
           for (int st = 0; st < 8 && ok; ++st) {
             uint32_t sa, fb;
-            if (!(ok = next_stage(sa, fb))) break;
+            if (!(ok = next_stage(sa, fb, w == 256 ? kStageTx : kStageTx / 2))) break;
             tma_load_2d_pair(sa, &tm_wn, fb, x, v0 + st * 64);
-            tma_load_2d_pair(sa + 8192, &tm_wn, fb, x + 64, v0 + st * 64);
+            if (w == 256) tma_load_2d_pair(sa + 8192, &tm_wn, fb, x + 64, v0 + st * 64);
           }
         }
         // dW jobs: h rows of the four tiles, 64 per stage, this CTA's 128 of the
         // job's 256 columns; the next unit's Z_a stages in between
         for (int j = 0; j < nJ && ok; ++j) {
-          const int x = j * 256 + static_cast<int>(prank) * 128;
+          const int w = job_w(j);
+          const int x = j * 256 + static_cast<int>(prank) * (w / 2);
           for (int st = 0; st < 8 && ok; ++st) {
             uint32_t sa, fb;
-            if (!(ok = next_stage(sa, fb))) break;
+            if (!(ok = next_stage(sa, fb, w == 256 ? kStageTx : kStageTx / 2))) break;
             const int row = t4[st >> 1] + (st & 1) * 64;
             tma_load_2d_pair(sa, &tm_h, fb, x, row);
-            tma_load_2d_pair(sa + 8192, &tm_h, fb, x + 64, row);
+            if (w == 256) tma_load_2d_pair(sa + 8192, &tm_h, fb, x + 64, row);
           }
           if (has_next)
-            for (int kb = 8 * j; kb < 8 * j + 8 && ok; ++kb) ok = load_z(kb, n_row0, n_v0);
+            for (int kb = 8 * j; kb < 8 * j + 8 && kb < nZ && ok; ++kb) ok = load_z(kb, n_row0, n_v0);
         }
       }
       if (leader) {
@@ -401,13 +407,14 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         for (int i = 0; i < nJ && ok; ++i) {
           if (!(ok = acc_free(jj))) break;
           const uint32_t d = tmem_base + kAccCol;
+          const uint32_t idesc = job_w(i) == 256 ? kIdescH : kIdescH128;
           for (int st = 0; st < 8 && ok; ++st) {   // 64 vocab rows x 128 columns per stage
             uint32_t sa;
             if (!(ok = wait_stage(sa))) break;
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
               const uint64_t bd = sdesc_sw128(sa + k * 2048, 8192, 1024);
-              umma_bf16_pair_ta(d, tmem_base + kGCol + 8u * static_cast<uint32_t>(st * 4 + k), bd, kIdescH,
+              umma_bf16_pair_ta(d, tmem_base + kGCol + 8u * static_cast<uint32_t>(st * 4 + k), bd, idesc,
                                 (st | k) != 0 ? 1u : 0u);
             }
             release_stage();
@@ -424,6 +431,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         for (int j = 0; j < nJ && ok; ++j) {
           if (!(ok = acc_free(jj))) break;
           const uint32_t d = tmem_base + kAccCol;
+          const uint32_t idesc = job_w(j) == 256 ? kIdescW : kIdescW128;
           for (int st = 0; st < 8 && ok; ++st) {   // 64 token rows x 128 columns per stage
             uint32_t sa;
             if (!(ok = wait_stage(sa))) break;
@@ -431,7 +439,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
             for (int k = 0; k < 4; ++k) {
               const uint64_t ad = sdesc_sw128(gw_base + (st * 4 + k) * 2048, kGWBlock, 1024);
               const uint64_t bd = sdesc_sw128(sa + k * 2048, 8192, 1024);
-              umma_bf16_pair(d, ad, bd, kIdescW, (st | k) != 0 ? 1u : 0u);
+              umma_bf16_pair(d, ad, bd, idesc, (st | k) != 0 ? 1u : 0u);
             }
             release_stage();
           }
@@ -442,7 +450,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
               if (!(ok = mbar_wait(smem_u32(&dhd_bar), unit_it & 1u, abort_flag, a.err))) break;
               tc_fence_after();
             }
-            for (int kb = 8 * j; kb < 8 * j + 8 && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
+            for (int kb = 8 * j; kb < 8 * j + 8 && kb < nZ && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
           }
         }
         if (ok && !has_next) ok = mbar_wait(smem_u32(&dhd_bar), unit_it & 1u, abort_flag, a.err);
@@ -549,7 +557,8 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       ++nbox;
     };
     // one job: copy the accumulator to registers, hand it back, then drain it
-    auto drain_job = [&](const CUtensorMap* map, int x0, int y, bool issue) -> bool {
+    // (this warp's 128 of its 256 columns)
+    auto drain_job256 = [&](const CUtensorMap* map, int x0, int y, bool issue) -> bool {
       if (!mbar_wait(smem_u32(&accf_bar), jj & 1u, abort_flag, a.err)) return false;
       tc_fence_after();
       const uint32_t taddr = tmem_base + lane_off + kAccCol + hf * 128;
@@ -567,6 +576,25 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       drain_slab(map, v2, xh + 64, y, issue);
       drain_slab(map, v3, xh + 96, y, issue);
       return true;
+    };
+    // the same for a 128-column last job (H % 256 == 128): 64 columns per warp
+    auto drain_job128 = [&](const CUtensorMap* map, int x0, int y, bool issue) -> bool {
+      if (!mbar_wait(smem_u32(&accf_bar), jj & 1u, abort_flag, a.err)) return false;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + lane_off + kAccCol + hf * 64;
+      float v0[32], v1[32];
+      tmem_ld32(taddr, v0);
+      tmem_ld32(taddr + 32, v1);
+      tc_fence_before();
+      mbar_arrive_cluster_relaxed(acce_lead);
+      ++jj;
+      const int xh = x0 + hf * 64;
+      drain_slab(map, v0, xh, y, issue);
+      drain_slab(map, v1, xh + 32, y, issue);
+      return true;
+    };
+    auto drain_job = [&](const CUtensorMap* map, int x0, int y, bool issue, int w) -> bool {
+      return w == 256 ? drain_job256(map, x0, y, issue) : drain_job128(map, x0, y, issue);
     };
 
     UnitSeq seq;
@@ -618,14 +646,14 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       // the cluster's previous unit drained into the same rows
       order_drains(a.det_bands > 0);
       const int dh_row = own_row0 + q * 32 + seq.dh_copy() * a.det_rows;
-      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 256, dh_row, !own_null);
+      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 256, dh_row, !own_null, job_w(i));
       // dW jobs: this CTA's 128 vocab rows (its quarter; in the quad slot's
       // copy under the deterministic schedule), 256 columns of H each; the
       // previous drains into these rows came from the previous group
       order_drains(seq.group_start());
       const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
       const int dw_row = vrow + seq.dw_copy() * a.det_vrows;
-      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 256, dw_row, vrow < V);
+      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 256, dw_row, vrow < V, job_w(j));
       ++unit_it;
     }
     if (lane == 0) bulk_wait_group<0>();

@@ -127,7 +127,7 @@ cudaError_t launch_sum_copies(const float* copies, int64_t n, int n_copies, floa
 // lmhead_fwd.cu
 cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,
                               cudaStream_t s);
-// lmhead_bwd4.cu (clusters of two CTA pairs; H % 256 == 0)
+// lmhead_bwd4.cu (clusters of two CTA pairs; H % 128 == 0)
 int lmhead_bwd_quad_clusters(int n_sm);       // clusters one raster launch runs
 int lmhead_bwd_quad_det_clusters(int n_sm);   // clusters of the deterministic schedule (multiple of 4)
 // host: count kernels the library enqueued (molt_kernel_launches)

@@ -224,7 +224,8 @@ def test_bad_options_rejected():
 # (5000, 256, 9000): about 7 token quads (two groups of four) and 18 vocab
 # blocks (two per residue class on a GB300), so both reduction orders of the
 # schedule have more than one step
-DET_SHAPES = [(1000, 256, 5000), (513, 512, 4133), (640, 768, 2304), (1, 256, 7), (5000, 256, 9000)]
+DET_SHAPES = [(1000, 256, 5000), (513, 512, 4133), (640, 768, 2304), (1, 256, 7), (5000, 256, 9000),
+              (900, 384, 3000)]
 
 
 @pytest.mark.parametrize("T,H,V", DET_SHAPES)
@@ -279,7 +280,7 @@ def test_deterministic_mode_accumulates_and_combines_with_extended_terms():
     assert_grad_close(outs[0][1], ref["dH"], "dhidden (deterministic, extended terms)")
 
 
-def test_deterministic_mode_needs_h_multiple_of_256():
+def test_deterministic_mode_needs_h_multiple_of_128():
     rng = np.random.default_rng(4)
     h, W, x, m = random_problem(rng, 64, 192, 300)
     z = np.zeros(64, np.float32)

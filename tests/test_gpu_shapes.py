@@ -1,8 +1,8 @@
 """Seeded shape fuzzing of the policy-loss call against the fp64 oracle: token
 counts that leave 1-3 tiles of the last quad empty, vocabularies with ragged
 512-column blocks, H from 256 (two jobs per unit) upward, both the cluster
-backward (H % 256 == 0) and the single-CTA one, the deterministic schedule, and
-caller-provided workspaces."""
+backward (H % 128 == 0, a last 128-column job when H % 256 == 128) and the
+single-CTA one, the deterministic schedule, and caller-provided workspaces."""
 import ctypes
 
 import numpy as np
@@ -31,10 +31,10 @@ def _cases():
     rng = np.random.default_rng(2607)
     out = []
     for i in range(10):
-        H = int(rng.choice([256, 512, 768, 1024, 1280, 320]))
+        H = int(rng.choice([256, 384, 512, 640, 768, 896, 1024, 1280, 320]))
         T = int(rng.integers(1, 1800))
         V = int(rng.integers(1, 7000))
-        out.append((i, T, H, V, bool(i % 3 == 0) and H % 256 == 0))
+        out.append((i, T, H, V, bool(i % 3 == 0) and H % 128 == 0))
     return out
 
 
@@ -117,6 +117,35 @@ def test_vocab_split_with_side_kernel(V):
     assert n_split in (n_plain, n_plain + 1)
     if torch.cuda.get_device_properties(0).multi_processor_count == 152:
         assert n_split == n_plain + 1
+
+
+@pytest.mark.parametrize("H,V", [(384, 3000), (640, 4133), (896, 18986)])
+def test_half_width_last_job(H, V):
+    """H % 256 == 128: the cluster backward's last dH / dW job is 128 columns
+    wide.  Parity with the oracle on the raster schedule (V = 18986 also splits
+    the vocabulary with the side kernel) and on the deterministic one, which is
+    bitwise reproducible."""
+    T = 900
+    rng = np.random.default_rng(H + V)
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.25, w_std=0.05)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.28, H)
+    ref = O.policy_loss(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), m, 0.2, 0.28)
+    ref["_adv"] = adv.astype(np.float64)
+    args = (bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28)
+    runs = []
+    for det in (False, True, True):
+        out = molt.policy_loss_fwd_bwd_ex(*args, deterministic=det)
+        torch.cuda.synchronize()
+        assert molt.device_status() == 0
+        assert_loss_close(float(out["loss"].item()), ref)
+        assert_grad_close(np_(out["dhidden"]), ref["dH"], f"dhidden H={H} det={det}")
+        assert_grad_close(np_(out["dW"]), ref["dW"], f"dW H={H} det={det}")
+        runs.append(out)
+    for k in ("dhidden", "dW"):
+        np.testing.assert_array_equal(np_(runs[1][k]).view(np.uint8), np_(runs[2][k]).view(np.uint8), err_msg=k)
 
 
 def test_caller_workspace_and_too_small_workspace():
