@@ -171,6 +171,13 @@ molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, c
  * The [T,V] logits and gradients never reach global memory: each vocab tile is
  * recomputed on chip in the backward pass and fed to the dhidden / dW tensor-
  * core products from shared memory.
+ * Streams: all work is ordered on `stream`.  Part of the backward may run on an
+ * internal lowest-priority stream of the library (one per device and caller
+ * stream, created on the first such call), forked from `stream` and joined
+ * back to it with events before the call's later work, so nothing needs to be
+ * synchronised by the caller.  The call can be captured into a CUDA graph;
+ * the side stream is only used under capture if an earlier uncaptured call on
+ * the same stream created it.
  */
 size_t molt_policy_loss_workspace_bytes(int64_t T, int64_t H, int64_t V);
 molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,
