@@ -211,18 +211,21 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
  *   gate_lo, gate_hi   acceptance band of the geometric-mean ratio,
  *                 0 <= gate_lo <= gate_hi (gate_hi may be +inf)
  *   deterministic 1: dW and dhidden are bitwise reproducible for the same inputs
- *                 on the same device (no paper counterpart).  The backward then
- *                 fixes the order of every partial-sum reduction: each of its C
- *                 clusters (a multiple of 4) owns one slot of every group of
- *                 four 512-token quads and every (C/4)-th 512-column vocabulary
- *                 block; each dW element is reduced by one warp, in group order,
- *                 into the fp32 dW copy of its quad slot (4 copies), each
- *                 dhidden row, in block order, into one of C/4 fp32 copies, and
- *                 final passes sum the copies in copy order.  Needs H % 128 == 0
- *                 (MOLT_ERR_UNSUPPORTED_SHAPE otherwise) and the workspace of
- *                 molt_policy_loss_workspace_bytes_ex (C/4 [T, H] and four
- *                 [V, H] fp32 copies: C = 36 on a GB300).  0: reduce-adds in
- *                 arrival order (results agree to fp32 rounding).
+ *                 (no paper counterpart).  The backward then fixes the order of
+ *                 every partial-sum reduction: the partial products of a
+ *                 512-token quad x 512-column vocabulary block are reduce-added
+ *                 into dW in token-quad order and into dhidden in vocabulary
+ *                 block order, each [32 x 128] slab waiting its turn on a
+ *                 counter in the workspace.  The order does not depend on the
+ *                 number C of clusters the backward runs (a multiple of 4; C =
+ *                 36 on a GB300; the environment variable MOLT_DET_CLUSTERS
+ *                 may lower it).  The C clusters wait on one another, so they
+ *                 must be resident together: with other work occupying SMs for
+ *                 seconds the waits time out (MOLT_DEV_TIMEOUT; nothing hangs).
+ *                 Needs H % 128 == 0 (MOLT_ERR_UNSUPPORTED_SHAPE otherwise) and
+ *                 the workspace of molt_policy_loss_workspace_bytes_ex (the
+ *                 raster's plus the counters).  0: reduce-adds in arrival order
+ *                 (results agree to fp32 rounding).
  */
 typedef struct {
   float kl_coef;

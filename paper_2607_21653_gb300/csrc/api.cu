@@ -2,6 +2,7 @@
 // layout, TMA tensor maps and the launch sequence of each entry point.
 #include <atomic>
 #include <cstdint>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -129,13 +130,30 @@ int choose_splits(int64_t Tcap, int64_t V, int n_sm) {
 }
 
 struct Layout {
-  size_t counts, row_map, pos, tok_p, b_p, adv_p, h_p, part, zx, lse, coef, tile_flag, tile_list, red, dh32, dwc;
+  size_t counts, row_map, pos, tok_p, b_p, adv_p, h_p, part, zx, lse, coef, tile_flag, tile_list, red, dh32, turns;
   size_t lp_p, ent_p, ecoef, mu, gate_p, total;
 };
 
 constexpr size_t kNoRegion = ~size_t(0);   // a Layout region that is not allocated
 
-Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd, int dh_copies = 1, int dw_copies = 0) {
+// turn counters of the deterministic schedule: an abort word (padded to 64
+// words), then [token quads, H jobs, 32] for dhidden and [vocab blocks, H jobs,
+// 32] for dW
+struct TurnLayout {
+  int64_t dh_off, dw_off, words;
+};
+TurnLayout turn_layout(int64_t Tcap, int64_t H, int64_t V) {
+  const int64_t n_jobs = (H + 255) / 256;
+  const int64_t n_quads = (Tcap / kTileM + 3) / 4;
+  const int64_t n_blocks = (V + 511) / 512;
+  TurnLayout t;
+  t.dh_off = 64;
+  t.dw_off = t.dh_off + n_quads * n_jobs * 32;
+  t.words = t.dw_off + n_blocks * n_jobs * 32;
+  return t;
+}
+
+Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd, bool det = false) {
   const int64_t Tcap = round_tiles(T);
   const int64_t ntile = Tcap / kTileM;
   Layout L{};
@@ -159,8 +177,8 @@ Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd, int dh_copi
   L.tile_flag = take(ntile * 4);
   L.tile_list = take(ntile * 4);
   L.red = take(ntile * kRedSlots * 8);
-  L.dh32 = with_bwd ? take(static_cast<size_t>(dh_copies) * Tcap * H * 4) : o;
-  L.dwc = (with_bwd && dw_copies > 0) ? take(static_cast<size_t>(dw_copies) * V * H * 4) : kNoRegion;
+  L.dh32 = with_bwd ? take(static_cast<size_t>(Tcap) * H * 4) : o;
+  L.turns = (with_bwd && det) ? take(static_cast<size_t>(turn_layout(Tcap, H, V).words) * 4) : kNoRegion;
   L.lp_p = with_bwd ? take(Tcap * 4) : o;
   L.ent_p = with_bwd ? take(Tcap * 4) : o;
   L.ecoef = with_bwd ? take(Tcap * 4) : o;
@@ -188,7 +206,7 @@ Workspace carve(void* base, const Layout& L) {
   w.tile_list = reinterpret_cast<int32_t*>(p + L.tile_list);
   w.red = reinterpret_cast<double*>(p + L.red);
   w.dh32 = reinterpret_cast<float*>(p + L.dh32);
-  w.dwc = L.dwc != kNoRegion ? reinterpret_cast<float*>(p + L.dwc) : nullptr;
+  w.turns = L.turns != kNoRegion ? reinterpret_cast<uint32_t*>(p + L.turns) : nullptr;
   w.lp_p = reinterpret_cast<float*>(p + L.lp_p);
   w.ent_p = reinterpret_cast<float*>(p + L.ent_p);
   w.ecoef = reinterpret_cast<float*>(p + L.ecoef);
@@ -414,12 +432,18 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   }
   const int64_t Tcap = round_tiles(T);
   const int S = choose_splits(Tcap, V, di->n_sm);
-  // deterministic schedule: n_det clusters (a multiple of 4), n_det / 4
-  // dhidden copies and one dW copy per quad slot
-  const int n_det = det ? lmhead_bwd_quad_det_clusters(di->n_sm) : 0;
+  // deterministic schedule: n_det clusters (a multiple of 4), all resident at
+  // once, whose reduce-adds take turns
+  int n_det = det ? lmhead_bwd_quad_det_clusters(di->n_sm) : 0;
   if (det && n_det < 4) return fail(MOLT_ERR_UNSUPPORTED_SHAPE, "deterministic mode needs 4 clusters of 4 CTAs");
-  const int n_bands = det ? n_det / 4 : 1;
-  const Layout L = layout(T, H, V, S, true, n_bands, det ? 4 : 0);
+  if (det) {
+    // MOLT_DET_CLUSTERS: fewer clusters (a multiple of 4); the results do not
+    // depend on the count
+    const char* env = std::getenv("MOLT_DET_CLUSTERS");
+    const int want = env ? std::atoi(env) : 0;
+    if (want >= 4 && want % 4 == 0 && want < n_det) n_det = want;
+  }
+  const Layout L = layout(T, H, V, S, true, det);
   Scratch sc;
   MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
   const Workspace w = carve(sc.ptr, L);
@@ -437,11 +461,8 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   // 64-row boxes of h: a dW stage of the cluster backward is 64 token rows
   CUtensorMap tm_h64;
   MOLT_TRY(make_tmap(&tm_h64, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, 64));
-  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, n_bands * Tcap, H, 32, 32));
-  if (det)
-    MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dwc, 4 * V, H, 32, 32));
-  else
-    MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
+  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
+  MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
   MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
   if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
   if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
@@ -462,11 +483,10 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   MOLT_LAUNCH(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, stats_ex_out, di->status, stream),
             "finalize");
   ev_stop(2, stream);
-  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(n_bands) * Tcap * H * sizeof(float), stream),
-            "memset dh32");
-  if (det)
-    MOLT_CUDA(cudaMemsetAsync(w.dwc, 0, static_cast<size_t>(4) * V * H * sizeof(float), stream), "memset dW copies");
-  else if (!accumulate_dW)
+  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
+  const TurnLayout tl = turn_layout(Tcap, H, V);
+  if (det) MOLT_CUDA(cudaMemsetAsync(w.turns, 0, static_cast<size_t>(tl.words) * 4, stream), "memset turns");
+  if (!accumulate_dW)
     MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
   BwdArgs ba{};
   ba.tok_p = w.tok_p;
@@ -481,8 +501,11 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   ba.dh32 = w.dh32;
   ba.dW = dW_out;
   ba.det_bands = n_det;
-  ba.det_rows = static_cast<int>(Tcap);
-  ba.det_vrows = static_cast<int>(V);
+  if (det) {
+    ba.det_abort = w.turns;
+    ba.det_dh_turns = w.turns + tl.dh_off;
+    ba.det_dw_turns = w.turns + tl.dw_off;
+  }
   if (opts && ex.entropy_coef != 0.f) {
     ba.ecoef = w.ecoef;
     ba.mu = w.mu;
@@ -530,13 +553,9 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
     }
   } else
     MOLT_LAUNCH(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
-  if (det)
-    MOLT_LAUNCH(launch_sum_copies(w.dwc, V * H, 4, dW_out, accumulate_dW != 0, di->n_sm, stream), "sum dW copies");
   ev_stop(3, stream);
   ev_start(4, stream);
-  MOLT_LAUNCH(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), n_bands, Tcap * H, dhidden_out, di->n_sm,
-                           stream),
-            "cast dh");
+  MOLT_LAUNCH(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
   ev_stop(4, stream);
   return MOLT_OK;
 }
@@ -690,11 +709,7 @@ size_t molt_policy_loss_workspace_bytes_ex(int64_t T, int64_t H, int64_t V, cons
   const DeviceInfo* di = device_info(&st);
   const int n_sm = di ? di->n_sm : 152;
   const int64_t Tcap = round_tiles(T);
-  int n_det = det ? lmhead_bwd_quad_det_clusters(n_sm) : 0;
-  if (det && n_det < 4) n_det = n_sm / 16 * 4;   // no device to query: all SMs in clusters of four
-  if (det && n_det < 4) return 0;
-  return layout(T, H, V, choose_splits(Tcap > 0 ? Tcap : kTileM, V, n_sm), true, det ? n_det / 4 : 1,
-                det ? 4 : 0).total;
+  return layout(T, H, V, choose_splits(Tcap > 0 ? Tcap : kTileM, V, n_sm), true, det).total;
 }
 
 molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, const int32_t* tokens,

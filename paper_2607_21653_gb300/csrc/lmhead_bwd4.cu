@@ -122,11 +122,11 @@ __device__ __forceinline__ QuadUnit quad_unit_of(int u, int n_tq, int n_vp, int 
 // number of clusters, a multiple of 4): cluster c takes quad slot s = c % 4 of
 // every group of four token quads and the vocab blocks m, m + det / 4, ... with
 // m = c / 4; it walks the groups in order and, inside a group, its blocks in
-// order.  Every dW element then receives its contributions from one cluster in
-// group order (each quad slot drains into its own dW copy), and every dhidden
-// row from one cluster per residue class m in block order (one dhidden copy per
-// class).  At any time the four clusters of a class work on the same vocab
-// block, as in the raster with groups of four quads.
+// order.  The four clusters of a class then work on the same vocab block, one
+// quad each, and the det / 4 classes of a slot on consecutive blocks of one
+// quad, as in the raster with groups of four quads; the reduce-adds into a dW
+// row take turns in quad order, those into a dhidden row in block order (see
+// the epilogue).
 struct UnitSeq {
   int n_tq, n_vp, n_q, group, det;
   int u;                     // raster position
@@ -158,11 +158,6 @@ struct UnitSeq {
   __device__ __forceinline__ QuadUnit cur() const {
     return det > 0 ? QuadUnit{4 * g + slot, b} : quad_unit_of(u, n_tq, n_vp, group);
   }
-  __device__ __forceinline__ int dh_copy() const { return det > 0 ? m : 0; }
-  __device__ __forceinline__ int dw_copy() const { return det > 0 ? slot : 0; }
-  // deterministic: the first of this cluster's units in its group (the previous
-  // contributions to its dW rows came from the previous group)
-  __device__ __forceinline__ bool group_start() const { return det > 0 && b == m; }
   __device__ __forceinline__ void advance() {
     if (det == 0) {
       u += n_q;
@@ -556,9 +551,40 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       if (lane == 0) bulk_commit_group();
       ++nbox;
     };
+    // Deterministic schedule: the reduce-adds into each [32 x 128] slab of an
+    // accumulator take turns.  The slabs of a quad's dhidden rows receive their
+    // contributions in vocab-block order, those of a block's dW rows in
+    // token-quad order, each from the warp of the same role in another cluster
+    // (the same rows and columns).  A turn counter per slab counts the
+    // contributions that have completed: a warp waits until it equals its own
+    // position (block or quad index), drains, and raises it once its
+    // reduce-adds have completed, at its next drain or the end of the unit, so
+    // that it does not wait for them in between.
+    uint32_t* pend = nullptr;   // counter to raise, and its new value
+    uint32_t pend_val = 0;
+    auto release_turn = [&]() {
+      if (pend != nullptr) {
+        if (lane == 0) {
+          bulk_wait_group<0>();
+          fence_proxy_async_global();
+          st_release_gpu(pend, pend_val);
+        }
+        __syncwarp();
+        pend = nullptr;
+      }
+    };
+    auto take_turn = [&](uint32_t* turn, uint32_t pos) -> bool {
+      int good = 1;
+      if (lane == 0) {
+        good = turn_wait(turn, pos, abort_flag, a.det_abort, a.err) ? 1 : 0;
+        fence_proxy_async_global();
+      }
+      return __shfl_sync(0xffffffffu, good, 0) != 0;
+    };
     // one job: copy the accumulator to registers, hand it back, then drain it
-    // (this warp's 128 of its 256 columns)
-    auto drain_job256 = [&](const CUtensorMap* map, int x0, int y, bool issue) -> bool {
+    // (this warp's 128 of its 256 columns); `turn` (deterministic schedule) is
+    // the slab's counter and `pos` this contribution's place in its order
+    auto drain_job256 = [&](const CUtensorMap* map, int x0, int y, bool issue, uint32_t* turn, uint32_t pos) -> bool {
       if (!mbar_wait(smem_u32(&accf_bar), jj & 1u, abort_flag, a.err)) return false;
       tc_fence_after();
       const uint32_t taddr = tmem_base + lane_off + kAccCol + hf * 128;
@@ -570,15 +596,21 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive_cluster_relaxed(acce_lead);
       ++jj;
+      release_turn();
+      if (turn != nullptr && !take_turn(turn, pos)) return false;
       const int xh = x0 + hf * 128;
       drain_slab(map, v0, xh, y, issue);
       drain_slab(map, v1, xh + 32, y, issue);
       drain_slab(map, v2, xh + 64, y, issue);
       drain_slab(map, v3, xh + 96, y, issue);
+      if (turn != nullptr) {
+        pend = turn;
+        pend_val = pos + 1;
+      }
       return true;
     };
     // the same for a 128-column last job (H % 256 == 128): 64 columns per warp
-    auto drain_job128 = [&](const CUtensorMap* map, int x0, int y, bool issue) -> bool {
+    auto drain_job128 = [&](const CUtensorMap* map, int x0, int y, bool issue, uint32_t* turn, uint32_t pos) -> bool {
       if (!mbar_wait(smem_u32(&accf_bar), jj & 1u, abort_flag, a.err)) return false;
       tc_fence_after();
       const uint32_t taddr = tmem_base + lane_off + kAccCol + hf * 64;
@@ -588,13 +620,26 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive_cluster_relaxed(acce_lead);
       ++jj;
+      release_turn();
+      if (turn != nullptr && !take_turn(turn, pos)) return false;
       const int xh = x0 + hf * 64;
       drain_slab(map, v0, xh, y, issue);
       drain_slab(map, v1, xh + 32, y, issue);
+      if (turn != nullptr) {
+        pend = turn;
+        pend_val = pos + 1;
+      }
       return true;
     };
-    auto drain_job = [&](const CUtensorMap* map, int x0, int y, bool issue, int w) -> bool {
-      return w == 256 ? drain_job256(map, x0, y, issue) : drain_job128(map, x0, y, issue);
+    auto drain_job = [&](const CUtensorMap* map, int x0, int y, bool issue, int w, uint32_t* turn,
+                         uint32_t pos) -> bool {
+      return w == 256 ? drain_job256(map, x0, y, issue, turn, pos) : drain_job128(map, x0, y, issue, turn, pos);
+    };
+    // this warp's slab counters (deterministic schedule): [unit, job, CTA, warp]
+    const bool det = a.det_bands > 0;
+    const int slab = static_cast<int>(rank) * 8 + (warp - 2);
+    auto turn_of = [&](uint32_t* base, int unit, int job) -> uint32_t* {
+      return det ? base + (static_cast<size_t>(unit) * nJ + job) * 32 + slab : nullptr;
     };
 
     UnitSeq seq;
@@ -633,29 +678,23 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       tc_fence_before();
       mbar_arrive_cluster(tb_lead);
       mbar_arrive_cluster(gw_lead1);
-      // deterministic schedule: this warp's earlier reduce-adds into the same
-      // rows complete before the next ones are issued
-      auto order_drains = [&](bool needed) {
-        if (needed) {
-          if (lane == 0) bulk_wait_group<0>();
-          __syncwarp();
-        }
-      };
-      // dH jobs: this CTA's 128 token rows (in the class's copy of the
-      // accumulator under the deterministic schedule), 256 columns of H each;
-      // the cluster's previous unit drained into the same rows
-      order_drains(a.det_bands > 0);
-      const int dh_row = own_row0 + q * 32 + seq.dh_copy() * a.det_rows;
-      for (int i = 0; i < nJ && ok; ++i) ok = drain_job(&tm_dh, i * 256, dh_row, !own_null, job_w(i));
-      // dW jobs: this CTA's 128 vocab rows (its quarter; in the quad slot's
-      // copy under the deterministic schedule), 256 columns of H each; the
-      // previous drains into these rows came from the previous group
-      order_drains(seq.group_start());
+      // dH jobs: this CTA's 128 token rows, 256 columns of H each (in turn
+      // after the quad's earlier vocab blocks)
+      const int dh_row = own_row0 + q * 32;
+      for (int i = 0; i < nJ && ok; ++i)
+        ok = drain_job(&tm_dh, i * 256, dh_row, !own_null, job_w(i), turn_of(a.det_dh_turns, un.tq, i),
+                       static_cast<uint32_t>(un.vp));
+      // dW jobs: this CTA's 128 vocab rows (its quarter), 256 columns of H
+      // each (in turn after the block's earlier token quads)
       const int vrow = v0 + static_cast<int>(rank) * 128 + q * 32;
-      const int dw_row = vrow + seq.dw_copy() * a.det_vrows;
-      for (int j = 0; j < nJ && ok; ++j) ok = drain_job(&tm_dw, j * 256, dw_row, vrow < V, job_w(j));
+      for (int j = 0; j < nJ && ok; ++j)
+        ok = drain_job(&tm_dw, j * 256, vrow, vrow < V, job_w(j), turn_of(a.det_dw_turns, un.vp, j),
+                       static_cast<uint32_t>(un.tq));
+      // the unit's last dW slab: the next quad's warp is waiting for it
+      release_turn();
       ++unit_it;
     }
+    release_turn();
     if (lane == 0) bulk_wait_group<0>();
     __syncwarp();
   }

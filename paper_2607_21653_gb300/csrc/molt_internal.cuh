@@ -31,8 +31,8 @@ struct Workspace {
   int32_t* tile_flag;   // [Tcap/128]
   int32_t* tile_list;   // [Tcap/128]
   double* red;          // [n_tiles * kRedSlots] per-tile partial sums
-  float* dh32;          // [copies, Tcap, H] fp32 dhidden accumulator(s) (loss call only)
-  float* dwc;           // [4, V, H] fp32 dW copies of the deterministic schedule, or nullptr
+  float* dh32;          // [Tcap, H] fp32 dhidden accumulator (loss call only)
+  uint32_t* turns;      // deterministic schedule: abort word + turn counters, or nullptr
   // extended objective (loss call only)
   float* lp_p;          // [Tcap] packed log-probs
   float* ent_p;         // [Tcap] packed entropies
@@ -72,10 +72,10 @@ struct BwdArgs {
   float* dh32;               // [Tcap, H] fp32 dhidden accumulator
   float* dW;                 // [V, H] fp32 dW
   int det_bands;             // 0: raster schedule; > 0: deterministic schedule on this many
-                             // clusters (a multiple of 4): det_bands / 4 dhidden copies and
-                             // 4 dW copies, one per quad slot
-  int det_rows;              // rows between the dhidden accumulator copies (Tcap)
-  int det_vrows;             // rows between the dW copies (V)
+                             // clusters (a multiple of 4), reduce-adds taking turns
+  uint32_t* det_abort;       // deterministic: set once any turn wait gives up (zeroed per call)
+  uint32_t* det_dh_turns;    // deterministic: [token quads, H jobs, 32] counters, blocks done
+  uint32_t* det_dw_turns;    // deterministic: [vocab blocks, H jobs, 32] counters, quads done
   unsigned* err;
 };
 
@@ -116,13 +116,8 @@ cudaError_t launch_merge_stats_ex(int Tcap, int V, int n_split, const Workspace&
 cudaError_t launch_seq_gate(int T, int Tcap, const LossEx& ex, const Workspace& ws, unsigned* err, cudaStream_t s);
 cudaError_t launch_loss_rows_ex(int Tcap, double denom, float clip_lo, float clip_hi, const LossEx& ex,
                                 const Workspace& ws, float* tokloss_out, cudaStream_t s);
-// dhidden_out[t] = bf16(sum over the n_copies accumulator copies, in copy order)
-cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, int n_copies, int64_t copy_stride, uint16_t* dh_out,
-                           int n_sm, cudaStream_t s);
-// out = (accumulate ? out : 0) + copies[0] + ... + copies[n_copies - 1], in that
-// order (n elements, a multiple of 4; copies n elements apart)
-cudaError_t launch_sum_copies(const float* copies, int64_t n, int n_copies, float* out, bool accumulate, int n_sm,
-                              cudaStream_t s);
+// dhidden_out[t] = bf16(the fp32 accumulator row of t)
+cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s);
 
 // lmhead_fwd.cu
 cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,

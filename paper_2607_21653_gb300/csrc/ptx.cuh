@@ -125,6 +125,48 @@ __device__ __forceinline__ void bulk_wait_group() {
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+// orders this thread's generic-proxy accesses of global memory with its
+// async-proxy (TMA) ones
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_relaxed_gpu(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release_gpu(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Bounded wait until the counter *turn (raised by other CTAs with release
+// stores) reaches `target`.  Gives up at once when this CTA or the call has
+// aborted, and after kWaitTimeoutNs; a timeout raises both abort flags and the
+// device error word.
+__device__ __forceinline__ bool turn_wait(const uint32_t* turn, uint32_t target, volatile int* abort_flag,
+                                          uint32_t* call_abort, unsigned* err) {
+  if (ld_acquire_gpu(turn) >= target) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1; i < kWaitMaxPolls; ++i) {
+    __nanosleep(64);
+    if (ld_acquire_gpu(turn) >= target) return true;
+    if ((i & 15u) == 0u) {
+      if (*abort_flag || ld_relaxed_gpu(call_abort) != 0u) {
+        *abort_flag = 1;
+        return false;
+      }
+      if (globaltimer_ns() - t0 > kWaitTimeoutNs) break;
+    }
+  }
+  *abort_flag = 1;
+  atomicExch(call_abort, 1u);
+  if (err) atomicOr(err, kDevErrTimeout);
+  return false;
+}
 __device__ __forceinline__ uint64_t l2_policy_evict_last() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));

@@ -564,10 +564,9 @@ __global__ void __launch_bounds__(1024) finalize_kernel(double denom, int32_t* _
   if (threadIdx.x == 0) counts[1] = total;
 }
 
-// dhidden_out[t] = bf16(sum_c dh32[c][pos[t]]) for active rows (copies summed
-// in order c = 0, 1, ...), 0 for masked rows
+// dhidden_out[t] = bf16(dh32[pos[t]]) for active rows, 0 for masked rows
 __global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __restrict__ pos, int T, int H,
-                               int n_copies, int64_t copy_stride, uint16_t* __restrict__ out) {
+                               uint16_t* __restrict__ out) {
   const int vpr = H / 8;
   const int64_t total = (int64_t)T * vpr;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
@@ -576,13 +575,7 @@ __global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __
     uint4 o = make_uint4(0, 0, 0, 0);
     if (k >= 0) {
       const float4* src = reinterpret_cast<const float4*>(dh32 + (int64_t)k * H) + 2 * v;
-      float4 a = src[0], c = src[1];
-      for (int cp = 1; cp < n_copies; ++cp) {
-        const float4* s2 = reinterpret_cast<const float4*>(dh32 + cp * copy_stride + (int64_t)k * H) + 2 * v;
-        const float4 a2 = s2[0], c2 = s2[1];
-        a.x += a2.x; a.y += a2.y; a.z += a2.z; a.w += a2.w;
-        c.x += c2.x; c.y += c2.y; c.z += c2.z; c.w += c2.w;
-      }
+      const float4 a = src[0], c = src[1];
       o.x = pack_bf16x2(a.x, a.y);
       o.y = pack_bf16x2(a.z, a.w);
       o.z = pack_bf16x2(c.x, c.y);
@@ -593,22 +586,6 @@ __global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __
 }
 
 }  // namespace
-
-// deterministic dW: the quad slots' copies summed in slot order
-__global__ void sum_copies_kernel(const float4* __restrict__ copies, int64_t n4, int n_copies, float4* out,
-                                  int accumulate) {
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n4; i += (int64_t)gridDim.x * blockDim.x) {
-    float4 a = accumulate ? out[i] : make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c = 0; c < n_copies; ++c) {
-      const float4 v = copies[c * n4 + i];
-      a.x += v.x;
-      a.y += v.y;
-      a.z += v.z;
-      a.w += v.w;
-    }
-    out[i] = a;
-  }
-}
 
 cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
                                     unsigned* err, cudaStream_t s) {
@@ -709,19 +686,9 @@ cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* 
   return cudaGetLastError();
 }
 
-cudaError_t launch_sum_copies(const float* copies, int64_t n, int n_copies, float* out, bool accumulate, int n_sm,
-                              cudaStream_t s) {
-  if (n <= 0) return cudaSuccess;
-  sum_copies_kernel<<<n_sm * 8, 256, 0, s>>>(reinterpret_cast<const float4*>(copies), n / 4, n_copies,
-                                             reinterpret_cast<float4*>(out), accumulate ? 1 : 0);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, int n_copies, int64_t copy_stride, uint16_t* dh_out,
-                           int n_sm, cudaStream_t s) {
+cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s) {
   if (T <= 0) return cudaSuccess;
-  cast_dh_kernel<<<n_sm * 8, 256, 0, s>>>(ws.dh32, ws.pos_of_row, T, H, n_copies < 1 ? 1 : n_copies, copy_stride,
-                                          dh_out);
+  cast_dh_kernel<<<n_sm * 8, 256, 0, s>>>(ws.dh32, ws.pos_of_row, T, H, dh_out);
   return cudaGetLastError();
 }
 

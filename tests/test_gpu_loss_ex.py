@@ -252,6 +252,38 @@ def test_deterministic_mode_is_bitwise_reproducible(T, H, V):
         abs(ref["loss"]), float(np.abs(ref["ratio"] * adv)[m != 0].sum() / ref["denom"]))
 
 
+@pytest.mark.parametrize("T,H,V", [(5000, 256, 9000), (2100, 640, 20000)])
+def test_deterministic_mode_does_not_depend_on_the_cluster_count(T, H, V, monkeypatch):
+    """The reduction order of the deterministic schedule is fixed by the turn
+    counters (dW in token-quad order, dhidden in vocab-block order), not by which
+    cluster runs which unit: 4, 8 and 16 clusters give the bits of the default
+    count, although units, timing and the clusters' waits all change.  (2100,
+    640, 20000) has a 128-column last job and 40 vocab blocks."""
+    rng = np.random.default_rng(T + H)
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.25, w_std=0.05)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.28, T + 5)
+    runs = {}
+    for n in (None, 16, 8, 4):
+        if n is None:
+            monkeypatch.delenv("MOLT_DET_CLUSTERS", raising=False)
+        else:
+            monkeypatch.setenv("MOLT_DET_CLUSTERS", str(n))
+        o = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28, deterministic=True)
+        torch.cuda.synchronize()
+        assert molt.device_status() == 0, n
+        runs[n] = (np_(o["dW"]).copy(), np_(o["dhidden"]).copy())
+    monkeypatch.delenv("MOLT_DET_CLUSTERS", raising=False)
+    for n in (16, 8, 4):
+        np.testing.assert_array_equal(runs[n][0].view(np.uint32), runs[None][0].view(np.uint32), err_msg=f"dW {n}")
+        np.testing.assert_array_equal(runs[n][1].view(np.uint16), runs[None][1].view(np.uint16), err_msg=f"dh {n}")
+    ref = O.policy_loss_ex(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), m, 0.2, 0.28)
+    assert_grad_close(runs[None][0], ref["dW"], "dW (deterministic)")
+    assert_grad_close(runs[None][1], ref["dH"], "dhidden (deterministic)")
+
+
 def test_deterministic_mode_accumulates_and_combines_with_extended_terms():
     rng = np.random.default_rng(21)
     lengths = [300, 1, 64, 400, 35]
