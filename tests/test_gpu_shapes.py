@@ -229,3 +229,33 @@ def test_concurrent_calls_on_two_streams():
         np.testing.assert_array_equal(np_(a["logp"]), np_(c["logp"]))
         assert_grad_close(np_(c["dhidden"]), np_(a["dhidden"]).astype(np.float64), "dhidden on a second stream")
         assert_grad_close(np_(c["dW"]), np_(a["dW"]).astype(np.float64), "dW on a second stream")
+
+
+def test_deterministic_calls_on_two_streams():
+    """Two deterministic calls issued on two streams at once.  Their clusters
+    wait on one another's turns, so each launch needs all its clusters resident:
+    the launch enqueued first takes the SMs, the other's clusters start as its
+    clusters leave.  Each result equals the same problem run alone, bit for bit,
+    and no wait times out."""
+    probs = []
+    for i in range(2):
+        rng = np.random.default_rng(60 + i)
+        T, H, V = 3000, 512, 9000 + 1000 * i
+        h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
+        m[0] = 1
+        adv = rng.standard_normal(T).astype(np.float32)
+        b = behavior_from_oracle(O.widen_bf16(h), O.widen_bf16(W), x, 0.3, 0.2, 0.2, 70 + i)
+        probs.append((bf(h), bf(W), t(x), t(b), t(adv), t(m)))
+    alone = [molt.policy_loss_fwd_bwd_ex(*p, 0.2, 0.2, deterministic=True) for p in probs]
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    streams = [torch.cuda.Stream(), torch.cuda.Stream()]
+    together = []
+    for p, s in zip(probs, streams):
+        with torch.cuda.stream(s):
+            together.append(molt.policy_loss_fwd_bwd_ex(*p, 0.2, 0.2, deterministic=True, stream=s))
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    for a, c in zip(alone, together):
+        np.testing.assert_array_equal(np_(c["dW"]).view(np.uint32), np_(a["dW"]).view(np.uint32))
+        np.testing.assert_array_equal(np_(c["dhidden"]).view(np.uint16), np_(a["dhidden"]).view(np.uint16))
