@@ -239,3 +239,61 @@ def test_fullsize_extended_objective():
     live_seq = cnt > 0
     assert st["n_seq_rejected"] == int((~kept & live_seq).sum())
     assert st["n_tokens_rejected"] == int((act & ~kept[seq]).sum())
+
+
+def test_fullsize_whole_ragged_window_in_one_call():
+    """The ragged configuration's first 16 microbatches (1,048,576 tokens, H =
+    5120) in one call: T x H = 5.4e9 elements, past 2^32, so every row offset
+    of the packing, the backward and the casts needs 64-bit arithmetic.
+    Sampled rows (random active rows across the whole window plus one tile near
+    its end) against the oracle, and the whole-call properties of the
+    full-size tests, evaluated in row chunks."""
+    w = make_workload("ragged", T=16 * 65536)
+    assert w.T == 16 * 65536 and w.T * w.H > 2 ** 32
+    rng = np.random.default_rng(4321)
+    act_idx = np.nonzero(w.mask)[0]
+    rows = np.unique(np.concatenate([rng.choice(act_idx, size=N_RANDOM_ROWS, replace=False),
+                                     act_idx[-(act_idx.size % 128 + 128):][:128]]))
+    assert rows.max() * w.H > 2 ** 32
+    W64 = _w64(w)
+    h_c = O.widen_bf16(w.hidden[rows])          # the sampled rows only (rows are independent)
+    x_c = w.tokens[rows]
+    lp_c, _ = O.token_logprobs(h_c, W64, x_c, None, rows=np.arange(rows.size))
+    b = rng.normal(-np.log(w.V) - 1.0, 1.0, w.T)
+    b[rows] = lp_c + boundary_safe_noise(rng, rows.size, w.behavior_sigma, w.eps_lo, w.eps_hi,
+                                         2.5 * BOUNDARY_DELTA)
+    b = b.astype(np.float32)
+    adv = O.broadcast_advantages(O.group_advantages(w.rewards, w.group_ids), w.resp_of_token)
+    D = float(w.extra["window_denominator"])
+    hid = bf(w.hidden)
+    Wd = bf(w.weight)
+    out = molt.policy_loss_fwd_bwd(hid, Wd, t(w.tokens), t(b), t(adv.astype(np.float32)), t(w.mask), w.eps_lo,
+                                   w.eps_hi, denom=D)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    ref = O.policy_loss_rows(h_c, W64, x_c, b[rows].astype(np.float64), adv[rows].astype(np.float64),
+                             w.mask[rows], w.eps_lo, w.eps_hi, D, np.arange(rows.size))
+    lp, ent, tl = np_(out["logp"]), np_(out["entropy"]), np_(out["token_loss"])
+    assert np.abs(lp[rows] - ref["logp"]).max() <= LOGP_ATOL
+    assert np.abs(ent[rows] - ref["entropy"]).max() <= LOGP_ATOL
+    np.testing.assert_allclose(tl[rows], ref["token_loss"], rtol=5e-3, atol=1e-6)
+    dh = out["dhidden"]
+    assert_grad_close(np_(dh[torch.from_numpy(rows).to(dh.device)]), ref["dH"], "dhidden (sampled rows)")
+    assert np.abs(ref["dH"]).max() > 0, "the sampled rows must carry a gradient"
+    act = w.mask != 0
+    assert (lp[~act] == 0).all() and (tl[~act] == 0).all()
+    masked = torch.from_numpy(np.nonzero(~act)[0]).to(dh.device)
+    assert masked.numel() > 0 and int(torch.count_nonzero(dh[masked]).item()) == 0
+    L_tok = float(tl.astype(np.float64).sum() / D)
+    assert abs(float(out["loss"].item()) - L_tok) <= 1e-5 * max(1e-3, abs(L_tok))
+    dW = out["dW"]
+    col = dW.double().sum(dim=0)
+    col_abs = dW.double().abs().sum(dim=0)
+    assert float((col.abs() / col_abs.clamp_min(1e-30)).max().item()) < 1e-3
+    lhs = scale = 0.0
+    for r0 in range(0, w.T, 65536):
+        d = (dh[r0:r0 + 65536].double() * hid[r0:r0 + 65536].double()).sum(dim=1)
+        lhs += float(d.sum().item())
+        scale += float(d.abs().sum().item())
+    rhs = float((dW.double() * Wd.double()).sum().item())
+    assert abs(lhs - rhs) <= 1e-2 * scale, (lhs, rhs, scale)
