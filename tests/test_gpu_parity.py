@@ -239,3 +239,75 @@ def test_policy_loss_deterministic():
     o2 = molt.policy_loss_fwd_bwd(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2)
     assert float(o1["loss"].item()) == float(o2["loss"].item())
     np.testing.assert_array_equal(np_(o1["logp"]), np_(o2["logp"]))
+
+
+@pytest.mark.parametrize("H,det", [(64, False), (256, False), (256, True)])
+def test_single_class_vocabulary(H, det):
+    """V = 1, the degenerate softmax: p = 1, so logp = entropy = 0 and g = coef (p -
+    1) = 0 (dW and dhidden vanish up to the rounding of p next to 1); the loss
+    is the surrogate of rho = exp(-b) alone."""
+    rng = np.random.default_rng(H + int(det))
+    T = 300
+    h, W, x, m = random_problem(rng, T, H, 1, mask_frac=0.2, w_std=0.05)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    b = rng.normal(0.0, 0.3, T).astype(np.float32)
+    out = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28, deterministic=det)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    assert np.abs(np_(out["logp"])).max() <= 1e-6 and np.abs(np_(out["entropy"])).max() <= 1e-6
+    ref = O.policy_loss(O.widen_bf16(h), O.widen_bf16(W), x, b.astype(np.float64), adv.astype(np.float64), m,
+                        0.2, 0.28)
+    ref["_adv"] = adv.astype(np.float64)
+    assert_loss_close(float(out["loss"].item()), ref)
+    coef = np.abs(ref["coef"])
+    h_max = float(np.abs(O.widen_bf16(h)).max())
+    w_max = float(np.abs(O.widen_bf16(W)).max())
+    assert np.abs(np_(out["dW"])).max() <= 1e-5 * coef.sum() * h_max
+    assert np.abs(np_(out["dhidden"]).astype(np.float64)).max() <= 1e-5 * coef.max() * w_max
+
+
+@pytest.mark.parametrize("H,det", [(192, False), (512, False), (512, True)])
+def test_zero_advantages_skip_every_tile(H, det):
+    """A = 0 on every token: every coefficient m c / D is 0, every backward tile
+    is skipped, and the loss, dW and dhidden are exactly zero while logp and
+    entropy still match the oracle."""
+    rng = np.random.default_rng(7 * H + int(det))
+    T, V = 900, 3000
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.2, w_std=0.05)
+    m[0] = 1
+    adv = np.zeros(T, np.float32)
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.2, 9)
+    dW = torch.full((V, H), 7.0, device="cuda")
+    out = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2, deterministic=det, dW=dW)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    assert float(out["loss"].item()) == 0.0
+    assert not np_(out["dW"]).any() and not np_(out["dhidden"]).any()
+    lp_ref, ent_ref = O.token_logprobs(h64, W64, x, m)
+    assert np.abs(np_(out["logp"]) - lp_ref).max() <= LOGP_ATOL
+    assert np.abs(np_(out["entropy"]) - ent_ref).max() <= LOGP_ATOL
+
+
+@pytest.mark.parametrize("det", [False, True])
+def test_largest_hidden_size(det):
+    """H = 65536, the largest supported: 1024 K-blocks per logit tile in the
+    forward, 2048 logit stages per vocab half and 256 dH / dW jobs per unit in
+    the backward."""
+    rng = np.random.default_rng(65536 + int(det))
+    T, H, V = 130, 65536, 300
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.1, w_std=0.01)
+    m[0] = 1
+    adv = rng.standard_normal(T).astype(np.float32)
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.28, 3)
+    ref = O.policy_loss(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), m, 0.2, 0.28)
+    ref["_adv"] = adv.astype(np.float64)
+    out = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28, deterministic=det)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    assert np.abs(np_(out["logp"]) - ref["logp"]).max() <= LOGP_ATOL
+    assert_loss_close(float(out["loss"].item()), ref)
+    assert_grad_close(np_(out["dhidden"]), ref["dH"], "dhidden (H = 65536)")
+    assert_grad_close(np_(out["dW"]), ref["dW"], "dW (H = 65536)")
