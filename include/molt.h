@@ -19,9 +19,15 @@
  *   - Workspace: calls that need scratch memory take (workspace, bytes).  The
  *     size comes from the matching *_workspace_bytes() query.  Passing NULL
  *     makes the call allocate and free it stream-ordered (cudaMallocAsync).
- *   - The library keeps no state between calls except cached device properties
- *     and the per-device status word; it is safe to call from several threads
- *     on different streams with different workspaces.
+ *   - The library keeps no state between calls except cached device
+ *     properties, the per-device status word, the kernel-launch counter, the
+ *     no-allocation forward's fixed scratch array, and, for the loss call's
+ *     vocabulary split, one side stream with a fork and a join event per
+ *     (device, caller stream), created on first use (at most 64, never while the
+ *     caller's stream is being captured) and kept for the life of the process.
+ *     It is safe to call from several threads on different streams with
+ *     different workspaces; calls sharing a stream must come from one thread at
+ *     a time (their launches would interleave on it).
  */
 #ifndef MOLT_H_
 #define MOLT_H_
