@@ -234,18 +234,27 @@ def _stream(stream=None):
 
 
 _ws_cache: dict = {}
+_WS_CACHE_MAX = 16
 
 
 def _workspace(nbytes: int, device, key: str, stream=None):
     """Workspace buffer from the torch caching allocator, reused per (device,
     call kind, stream): calls on one stream run in order and can share it, calls
-    on different streams may overlap and get their own."""
+    on different streams may overlap and get their own.  Each buffer is
+    allocated on the stream that uses it, so that when it is replaced by a
+    larger one or evicted (beyond 16 entries, oldest first) the allocator
+    reuses its memory only after that stream's pending work."""
     torch = _torch()
-    k = (str(device), key, _stream(stream))
-    buf = _ws_cache.get(k)
+    s = torch.cuda.current_stream(device) if stream is None else stream
+    k = (str(device), key, s.cuda_stream)
+    buf = _ws_cache.pop(k, None)
     if buf is None or buf.numel() < nbytes:
-        buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
-        _ws_cache[k] = buf
+        buf = None
+        with torch.cuda.stream(s):
+            buf = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+    _ws_cache[k] = buf                   # most recently used last
+    while len(_ws_cache) > _WS_CACHE_MAX:
+        _ws_cache.pop(next(iter(_ws_cache)))
     return buf
 
 
