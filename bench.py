@@ -572,7 +572,7 @@ def main():
     ap.add_argument("--microbatch", type=int, default=None,
                     help="microbatch of a windowed workload (ragged: default 1)")
     ap.add_argument("--deterministic", action="store_true",
-                    help="bitwise-reproducible dW / dhidden (ordered reductions, one dhidden copy per band)")
+                    help="bitwise-reproducible dW / dhidden (reduce-adds take turns in a fixed order)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
