@@ -500,7 +500,7 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   ba.tile_group = pair_bwd ? 4 : 16;
   ba.dh32 = w.dh32;
   ba.dW = dW_out;
-  ba.det_bands = n_det;
+  ba.det_clusters = n_det;
   if (det) {
     ba.det_abort = w.turns;
     ba.det_dh_turns = w.turns + tl.dh_off;

@@ -286,7 +286,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         return true;
       };
       UnitSeq seq;
-      seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_bands);
+      seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_clusters);
       if (seq.valid()) {
         const QuadUnit un = seq.cur();
         const int own_row0 = tile_of(un.tq, static_cast<int>(rank)) * kTileM;
@@ -384,7 +384,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         return true;
       };
       UnitSeq seq;
-      seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_bands);
+      seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_clusters);
       if (seq.valid())
         for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb, kZaCol, smem_u32(&zfa_bar));
       for (; seq.valid() && ok; seq.advance()) {
@@ -636,14 +636,14 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       return w == 256 ? drain_job256(map, x0, y, issue, turn, pos) : drain_job128(map, x0, y, issue, turn, pos);
     };
     // this warp's slab counters (deterministic schedule): [unit, job, CTA, warp]
-    const bool det = a.det_bands > 0;
+    const bool det = a.det_clusters > 0;
     const int slab = static_cast<int>(rank) * 8 + (warp - 2);
     auto turn_of = [&](uint32_t* base, int unit, int job) -> uint32_t* {
       return det ? base + (static_cast<size_t>(unit) * nJ + job) * 32 + slab : nullptr;
     };
 
     UnitSeq seq;
-    seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_bands);
+    seq.init(quad, n_quads, n_tq, n_vp, a.tile_group, a.det_clusters);
     for (; seq.valid() && ok; seq.advance()) {
       const QuadUnit un = seq.cur();
       const bool own_null = 4 * un.tq + static_cast<int>(rank) >= n_tiles;
@@ -755,9 +755,9 @@ cudaError_t launch_lmhead_bwd_quad(const CUtensorMap& tm_hz, const CUtensorMap& 
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
   if (e != cudaSuccess) return e;
   int clusters = lmhead_bwd_quad_clusters(n_sm);
-  if (a.det_bands > 0) {
-    if (a.det_bands > clusters || a.det_bands % 4 != 0) return cudaErrorInvalidValue;
-    clusters = a.det_bands;
+  if (a.det_clusters > 0) {
+    if (a.det_clusters > clusters || a.det_clusters % 4 != 0) return cudaErrorInvalidValue;
+    clusters = a.det_clusters;
   }
   if (ent)
     lmhead_bwd_quad_kernel<true>

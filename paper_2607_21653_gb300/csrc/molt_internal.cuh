@@ -71,7 +71,7 @@ struct BwdArgs {
   const float* mu;           // sum_v p_v z_v per row (with ecoef)
   float* dh32;               // [Tcap, H] fp32 dhidden accumulator
   float* dW;                 // [V, H] fp32 dW
-  int det_bands;             // 0: raster schedule; > 0: deterministic schedule on this many
+  int det_clusters;          // 0: raster schedule; > 0: deterministic schedule on this many
                              // clusters (a multiple of 4), reduce-adds taking turns
   uint32_t* det_abort;       // deterministic: set once any turn wait gives up (zeroed per call)
   uint32_t* det_dh_turns;    // deterministic: [token quads, H jobs, 32] counters, blocks done
