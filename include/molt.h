@@ -81,6 +81,14 @@ int molt_version(void);
  * enqueue).  For launch accounting in benchmarks and tests. */
 uint64_t molt_kernel_launches(void);
 
+/* Self-test of the device-side wait bound (no paper counterpart).  One warp
+ * waits, exactly as the deterministic backward's turn waits do, on a counter
+ * that nothing raises: the wait gives up after its time limit (about 4 s),
+ * sets MOLT_DEV_TIMEOUT in the status word and the kernel returns, leaving the
+ * context usable.  Asynchronous on `stream` (scratch from cudaMallocAsync);
+ * read the outcome with molt_device_status. */
+molt_status molt_selftest_wait_timeout(cudaStream_t stream);
+
 /* Synchronises `stream`, returns the current device's status word in *flags
  * (MOLT_DEV_* bits) and clears it.  Returns the molt_status of the highest
  * priority set bit (MOLT_OK if none). */

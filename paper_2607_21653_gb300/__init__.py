@@ -110,6 +110,7 @@ def load():
         "molt_version": (I32, []),
         "molt_kernel_launches": (ctypes.c_uint64, []),
         "molt_device_status": (I32, [P, ctypes.POINTER(ctypes.c_uint32)]),
+        "molt_selftest_wait_timeout": (I32, [P]),
         "molt_group_advantages": (I32, [P, P, I64, D, P, P]),
         "molt_advantages": (I32, [P, P, I64, I32, D, P, P]),
         "molt_broadcast_advantages": (I32, [P, P, I64, I64, P, P]),
@@ -265,6 +266,13 @@ def device_status(stream=None) -> int:
     if st not in (0, 3, 4, 6, 8):
         _check(st)
     return int(flags.value)
+
+
+def selftest_wait_timeout(stream=None) -> None:
+    """Enqueue the wait self-test (molt_selftest_wait_timeout): a bounded device
+    wait on a counter nothing raises, which gives up after about 4 s and sets
+    the timeout bit; read it with device_status()."""
+    _check(load().molt_selftest_wait_timeout(_stream(stream)))
 
 
 def kernel_launches() -> int:

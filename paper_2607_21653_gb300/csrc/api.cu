@@ -614,6 +614,23 @@ void molt_set_timing_events(cudaEvent_t* starts, cudaEvent_t* stops, int n) {
   t_ev_n = (starts && stops && n > 0) ? n : 0;
 }
 
+molt_status molt_selftest_wait_timeout(cudaStream_t stream) {
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  void* words = nullptr;
+  MOLT_CUDA(cudaMallocAsync(&words, 16, stream), "cudaMallocAsync");
+  cudaError_t e = cudaMemsetAsync(words, 0, 16, stream);
+  if (e == cudaSuccess) {
+    e = molt::launch_wait_selftest(static_cast<uint32_t*>(words), di->status, stream);
+    if (e == cudaSuccess) molt::note_launches(1);
+  }
+  const cudaError_t e_free = cudaFreeAsync(words, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "wait self-test");
+  if (e_free != cudaSuccess) return cuda_fail(e_free, "cudaFreeAsync");
+  return MOLT_OK;
+}
+
 molt_status molt_device_status(cudaStream_t stream, uint32_t* flags) {
   if (!flags) return fail(MOLT_ERR_INVALID_ARG, "flags is NULL");
   molt_status st;

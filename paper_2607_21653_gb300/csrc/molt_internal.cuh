@@ -96,6 +96,8 @@ molt_status encode_tmap_2d(CUtensorMap* m, CUtensorMapDataType dt, int elem_byte
                            uint64_t cols, uint32_t box_cols, uint32_t box_rows);
 
 // rows.cu
+// one bounded turn wait on a counter nothing raises (words: 3 zeroed uint32)
+cudaError_t launch_wait_selftest(uint32_t* words, unsigned* err, cudaStream_t s);
 cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
                                     unsigned* err, cudaStream_t s);
 cudaError_t launch_advantages(const float* rewards, const int32_t* gids, int n, int estimator, double eps,

@@ -587,6 +587,22 @@ __global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __
 
 }  // namespace
 
+// words[0]: the call's abort word, words[1]: a counter nothing raises,
+// words[2]: 1 if the wait returned true, 2 if it gave up
+__global__ void wait_selftest_kernel(uint32_t* words, unsigned* err) {
+  __shared__ int abort_sh;
+  if (threadIdx.x == 0) {
+    abort_sh = 0;
+    volatile int* abort_flag = &abort_sh;
+    words[2] = turn_wait(words + 1, 1u, abort_flag, words, err) ? 1u : 2u;
+  }
+}
+
+cudaError_t launch_wait_selftest(uint32_t* words, unsigned* err, cudaStream_t s) {
+  wait_selftest_kernel<<<1, 32, 0, s>>>(words, err);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_group_advantages(const float* rewards, const int32_t* gids, int n, double eps, float* out,
                                     unsigned* err, cudaStream_t s) {
   return launch_advantages(rewards, gids, n, kAdvGrpo, eps, out, err, s);
