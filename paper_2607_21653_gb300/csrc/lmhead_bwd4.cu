@@ -192,7 +192,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) uint64_t full_bar[kStages];   // pair leader: both CTAs' bytes land here
   __shared__ __align__(8) uint64_t empty_bar[kStages];  // both CTAs of the pair
   __shared__ __align__(8) uint64_t accf_bar;            // both CTAs of the pair: accumulator full
-  __shared__ __align__(8) uint64_t acce_bar;            // pair leader: 512 epilogue arrivals (copied out)
+  __shared__ __align__(8) uint64_t acce_bar;            // pair leader: one arrival per epilogue warp of the pair (copied out)
   __shared__ __align__(8) uint64_t zfa_bar;             // every CTA: Z_a done in both pairs (2 commits)
   __shared__ __align__(8) uint64_t zfb_bar;             // every CTA: Z_b done in both pairs (2 commits)
   __shared__ __align__(8) uint64_t tb_bar;              // pair leader: Z_b read, g_b in TMEM (both CTAs' epilogues)
@@ -220,7 +220,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&empty_bar[s]), 1);
     }
     mbar_init(smem_u32(&accf_bar), 1);
-    mbar_init(smem_u32(&acce_bar), 2 * kEpiThreads);
+    mbar_init(smem_u32(&acce_bar), 2 * kEpiWarps);
     mbar_init(smem_u32(&zfa_bar), 2);
     mbar_init(smem_u32(&zfb_bar), 2);
     mbar_init(smem_u32(&tb_bar), 2 * kEpiThreads);
@@ -593,8 +593,11 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       tmem_ld32(taddr + 32, v1);
       tmem_ld32(taddr + 64, v2);
       tmem_ld32(taddr + 96, v3);
+      // every lane's TMEM reads are complete (wait::ld) and fenced; one
+      // arrival per warp hands the accumulator back
       tc_fence_before();
-      mbar_arrive_cluster_relaxed(acce_lead);
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster_relaxed(acce_lead);
       ++jj;
       release_turn();
       if (turn != nullptr && !take_turn(turn, pos)) return false;
@@ -618,7 +621,8 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       tmem_ld32(taddr, v0);
       tmem_ld32(taddr + 32, v1);
       tc_fence_before();
-      mbar_arrive_cluster_relaxed(acce_lead);
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster_relaxed(acce_lead);
       ++jj;
       release_turn();
       if (turn != nullptr && !take_turn(turn, pos)) return false;
