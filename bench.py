@@ -34,7 +34,25 @@ import sys
 import tempfile
 import time
 
+# torchrun starts every rank with OMP_NUM_THREADS=1.  The reference arm runs the
+# oracle on rank 0 alone, so there it gets every host core back; this has to
+# happen before numpy loads its BLAS.
+if "LOCAL_RANK" in os.environ and os.environ.get("RANK", "0") == "0" and "reference" in sys.argv[1:]:
+    for _k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ[_k] = str(os.cpu_count() or 1)
+
 import numpy as np
+
+
+def blas_threads():
+    """Threads numpy's BLAS runs the oracle's products on: the host cores,
+    unless a thread-count variable caps them."""
+    n = os.cpu_count() or 1
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        v = os.environ.get(k, "")
+        if v.isdigit() and int(v) > 0:
+            return min(n, int(v))
+    return n
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
@@ -248,7 +266,7 @@ def run_reference(args):
     ts = [step(i) for i in range(args.steps)]
     tot = sum(ts)
     value = rows_per_step * args.steps / tot
-    cores = os.cpu_count()
+    cores = blas_threads()
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
@@ -502,7 +520,7 @@ def run_ours(args):
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
         rate, nrows, secs = oracle_rows_rate(w, args.cpu_seconds)
-        cpu = {"value": rate, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+        cpu = {"value": rate, "unit": "tokens/s", "cores": blas_threads(), "kind": "oracle",
                "sample": f"{nrows} random active rows of the same batch (forward, dhidden rows, dW contribution), "
                          f"{secs:.1f} s, numpy fp64 BLAS on all host cores",
                "tiny_whole_tokens_per_s": oracle_tiny_whole_rate(),
