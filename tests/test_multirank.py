@@ -49,3 +49,18 @@ def test_single_rank_is_identity():
     assert bench.max_over_ranks(42.0, 1) == 42.0
     assert bench.rank_seed(None, 0, 1) is None
     assert bench.job_throughput(65536, 1, 10, 1000.0) == pytest.approx(655360.0)
+
+
+def test_cpu_baseline_reports_the_blas_threads(monkeypatch):
+    """cpu_baseline's `cores` is the thread count numpy's BLAS gets: the host
+    cores, capped by a thread-count variable such as the OMP_NUM_THREADS=1 that
+    torchrun gives every rank."""
+    import bench
+    for k in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        monkeypatch.delenv(k, raising=False)
+    n = os.cpu_count() or 1
+    assert bench.blas_threads() == n
+    monkeypatch.setenv("OMP_NUM_THREADS", "1")
+    assert bench.blas_threads() == 1
+    monkeypatch.setenv("OPENBLAS_NUM_THREADS", str(n + 7))
+    assert bench.blas_threads() == n
