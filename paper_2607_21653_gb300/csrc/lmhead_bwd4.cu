@@ -195,6 +195,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
   __shared__ __align__(8) uint64_t acce_bar;            // pair leader: one arrival per epilogue warp of the pair (copied out)
   __shared__ __align__(8) uint64_t zfa_bar;             // every CTA: Z_a done in both pairs (2 commits)
   __shared__ __align__(8) uint64_t zfb_bar;             // every CTA: Z_b done in both pairs (2 commits)
+  __shared__ __align__(8) uint64_t zfo_bar;             // every CTA: Z_b done in its own pair (1 commit)
   __shared__ __align__(8) uint64_t tb_bar;              // pair leader: Z_b read, g_b in TMEM (both CTAs' epilogues)
   __shared__ __align__(8) uint64_t gw_bar;              // pair leader: both GW buffers of the pair full (all 4 CTAs)
   __shared__ __align__(8) uint64_t dhd_bar;             // pair leader: this unit's dH products done
@@ -223,6 +224,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
     mbar_init(smem_u32(&acce_bar), 2 * kEpiWarps);
     mbar_init(smem_u32(&zfa_bar), 2);
     mbar_init(smem_u32(&zfb_bar), 2);
+    mbar_init(smem_u32(&zfo_bar), 1);
     mbar_init(smem_u32(&tb_bar), 2 * kEpiThreads);
     mbar_init(smem_u32(&gw_bar), 4 * kEpiThreads);
     mbar_init(smem_u32(&dhd_bar), 1);
@@ -396,6 +398,7 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
         if (!(ok = acc_free(jj))) break;
         for (int kb = 0; kb < nZ && ok; ++kb) ok = z_block(kb, kZbCol, smem_u32(&zfb_bar));
         if (!ok) break;
+        umma_commit_pair_mc(smem_u32(&zfo_bar), pair_mask);
         // dH: A = g from TMEM (K = 512 vocab), B = W rows (MN-major)
         if (!(ok = mbar_wait_cluster(smem_u32(&tb_bar), unit_it & 1u, abort_flag, a.err))) break;
         tc_fence_after();
@@ -480,11 +483,27 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
     uint32_t jj = 0, nbox = 0, unit_it = 0;
     bool ok = true;
 
-    // z (32 columns at zaddr) -> g for vocab columns vc0 .. vc0+31 of the unit:
-    // packed into w (stored to TMEM by the caller) and into the GW buffer of the
-    // CTA that owns those columns
+    // g for vocab columns vc0 .. vc0+31 of the unit (packed in w) -> the GW
+    // buffer of the CTA that owns those columns
+    auto store_gw32 = [&](const uint32_t (&w)[16], int vc0) {
+      const int owner = vc0 >> 7;                 // vocab quarter -> CTA
+      const int cq = vc0 & 127;
+      const uint32_t off = static_cast<uint32_t>((cq >> 6) * kGWBlock) + gw_row;
+      const int cc0 = (cq & 63) >> 3;             // first 16-byte chunk in the row
+      const uint32_t dst = mapa_shared(gw_base, static_cast<uint32_t>(owner)) + off;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint32_t pos = static_cast<uint32_t>(((cc0 + i) ^ (r_in & 7)) * 16);
+        if (owner == static_cast<int>(rank))
+          st_shared_v4(gw_base + off + pos, w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+        else
+          st_shared_cluster_v4(dst + pos, w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
+      }
+    };
+    // z (32 columns at zaddr) -> g for vocab columns vc0 .. vc0+31 of the unit,
+    // packed into w (stored to TMEM by the caller), and into GW if to_gw
     auto convert32 = [&](uint32_t zaddr, uint32_t (&w)[16], int vc0, float coef, float ecoef, float mu, float lseL,
-                         int lx, int nvalid, bool live) {
+                         int lx, int nvalid, bool live, bool to_gw) {
       float v[32];
       tmem_ld32(zaddr, v);
       if (live) {
@@ -510,30 +529,18 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int j = 0; j < 16; ++j) w[j] = 0u;
       }
-      const int owner = vc0 >> 7;                 // vocab quarter -> CTA
-      const int cq = vc0 & 127;
-      const uint32_t off = static_cast<uint32_t>((cq >> 6) * kGWBlock) + gw_row;
-      const int cc0 = (cq & 63) >> 3;             // first 16-byte chunk in the row
-      const uint32_t dst = mapa_shared(gw_base, static_cast<uint32_t>(owner)) + off;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint32_t pos = static_cast<uint32_t>(((cc0 + i) ^ (r_in & 7)) * 16);
-        if (owner == static_cast<int>(rank))
-          st_shared_v4(gw_base + off + pos, w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
-        else
-          st_shared_cluster_v4(dst + pos, w[4 * i], w[4 * i + 1], w[4 * i + 2], w[4 * i + 3]);
-      }
+      if (to_gw) store_gw32(w, vc0);
     };
     // one logit half (256 columns of z at zcol, vocab vc_base ..): this warp
     // converts its 128 columns; both warps of the lane quarter read all their z
     // before either writes g over it (in place: column c -> c / 2)
     auto convert_half = [&](uint32_t zrow, uint32_t zcol, uint32_t gcol, int vc_base, float coef, float ecoef,
-                            float mu, float lseL, int lx, int nvalid, bool live) -> bool {
-      uint32_t w[4][16];
+                            float mu, float lseL, int lx, int nvalid, bool live, uint32_t (&w)[4][16],
+                            bool to_gw) -> bool {
 #pragma unroll
       for (int c = 0; c < 4; ++c)
         convert32(zrow + zcol + hf * 128 + 32 * c, w[c], vc_base + hf * 128 + 32 * c, coef, ecoef, mu, lseL, lx,
-                  nvalid, live);
+                  nvalid, live, to_gw);
       if (!pair_warps_sync()) return false;
 #pragma unroll
       for (int c = 0; c < 4; ++c) tmem_st16(zrow + gcol + hf * 64 + 16 * c, w[c]);
@@ -670,17 +677,25 @@ __global__ void __cluster_dims__(4, 1, 1) __launch_bounds__(kThreads, 1)
       // Z_a -> g of vocab 0..255: TMEM columns [0, 128), GW of CTAs 0 and 1
       if (!(ok = mbar_wait_cluster(smem_u32(&zfa_bar), unit_it & 1u, abort_flag, a.err))) break;
       tc_fence_after();
-      if (!(ok = convert_half(zrow, kZaCol, kGCol, 0, coef, ecoef, mu, lseL, lx, nvalid, live))) break;
+      uint32_t w[4][16];
+      if (!(ok = convert_half(zrow, kZaCol, kGCol, 0, coef, ecoef, mu, lseL, lx, nvalid, live, w, true))) break;
       fence_proxy_async_cluster();
       tc_fence_before();
       mbar_arrive_cluster(gw_lead0);
-      // Z_b -> g of vocab 256..511: TMEM columns [128, 256), GW of CTAs 2 and 3
-      if (!(ok = mbar_wait_cluster(smem_u32(&zfb_bar), unit_it & 1u, abort_flag, a.err))) break;
+      // Z_b -> g of vocab 256..511: TMEM columns [128, 256) as soon as this
+      // pair's Z_b is done; GW of CTAs 2 and 3 once both pairs' are
+      if (!(ok = mbar_wait_cluster(smem_u32(&zfo_bar), unit_it & 1u, abort_flag, a.err))) break;
       tc_fence_after();
-      if (!(ok = convert_half(zrow, kZbCol, kGCol + 128, 256, coef, ecoef, mu, lseL, lx, nvalid, live))) break;
-      fence_proxy_async_cluster();
+      if (!(ok = convert_half(zrow, kZbCol, kGCol + 128, 256, coef, ecoef, mu, lseL, lx, nvalid, live, w, false)))
+        break;
+      // the dH products need only g in TMEM and Z_b read out: a relaxed
+      // arrival after the TMEM fence; the GW stores follow, released on gw_bar
       tc_fence_before();
-      mbar_arrive_cluster(tb_lead);
+      mbar_arrive_cluster_relaxed(tb_lead);
+      if (!(ok = mbar_wait_cluster(smem_u32(&zfb_bar), unit_it & 1u, abort_flag, a.err))) break;
+#pragma unroll
+      for (int c = 0; c < 4; ++c) store_gw32(w[c], 256 + hf * 128 + 32 * c);
+      fence_proxy_async_cluster();
       mbar_arrive_cluster(gw_lead1);
       // dH jobs: this CTA's 128 token rows, 256 columns of H each (in turn
       // after the quad's earlier vocab blocks)
