@@ -58,6 +58,7 @@ an exact slice of policy_loss_ex.
 from __future__ import annotations
 
 import math
+from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
 
@@ -65,6 +66,7 @@ __all__ = [
     "widen_bf16", "group_advantages", "advantages", "ESTIMATORS", "broadcast_advantages", "logits_rows",
     "row_softmax_stats", "token_logprobs", "policy_loss", "policy_loss_rows",
     "clip_decision", "surrogate", "policy_loss_ex", "sequence_gate", "policy_loss_ex_rows",
+    "full_forward_rows", "dW_rows", "shard_partials", "merge_shard_partials",
 ]
 
 DEFAULT_ADV_EPS = 1e-6
@@ -472,3 +474,122 @@ def policy_loss_ex_rows(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, b
         out["coef"][pos] = coef
         out["dH"][pos] = g @ W
     return out
+
+
+# --------------------------------------------------------------------------- #
+# Whole-batch forward and sampled dW rows at the full vocabulary size
+# --------------------------------------------------------------------------- #
+def _row_stats_block(z: np.ndarray, x: np.ndarray):
+    """lse, logp of target x and entropy for each row of z (the definitions of
+    row_softmax_stats without returning the probabilities)."""
+    M = z.max(axis=1)
+    e = np.exp(z - M[:, None])
+    s = e.sum(axis=1)
+    lse = M + np.log(s)
+    logp = z[np.arange(z.shape[0]), x] - lse
+    # sum_v p_v z_v with p_v = e_v / s
+    ent = lse - (e * z).sum(axis=1) / s
+    return lse, logp, ent
+
+
+def full_forward_rows(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, rows: np.ndarray,
+                      block: int = 1024, workers: int = 1):
+    """lse, logp and entropy (fp64) of every given row against the whole
+    vocabulary: z = h W^T, lse = max + log sum exp(z - max), logp = z[x] - lse,
+    entropy = lse - sum_v p_v z_v (the definitions of Sec. 4.5's recomputed
+    probabilities, as in row_softmax_stats).  One matmul per block of rows;
+    the per-row reductions of a block may run on `workers` threads, each over
+    its own rows, which changes no per-row result."""
+    rows = np.asarray(rows)
+    n = rows.shape[0]
+    lse = np.zeros(n)
+    logp = np.zeros(n)
+    ent = np.zeros(n)
+    x_all = np.asarray(tokens)
+    pool = ThreadPoolExecutor(max_workers=workers) if workers > 1 else None
+    try:
+        for b0 in range(0, n, block):
+            sl = np.arange(b0, min(n, b0 + block))
+            t = rows[sl]
+            z = logits_rows(hidden[t], W)
+            x = x_all[t]
+            if pool is None:
+                lse[sl], logp[sl], ent[sl] = _row_stats_block(z, x)
+                continue
+            parts = np.array_split(np.arange(sl.shape[0]), workers)
+            res = list(pool.map(lambda p: _row_stats_block(z[p], x[p]), [p for p in parts if p.size]))
+            for p, (a, b, c) in zip([p for p in parts if p.size], res):
+                lse[sl[p]], logp[sl[p]], ent[sl[p]] = a, b, c
+    finally:
+        if pool is not None:
+            pool.shutdown()
+    return lse, logp, ent
+
+
+def dW_rows(hidden: np.ndarray, W: np.ndarray, tokens: np.ndarray, lse: np.ndarray, coef: np.ndarray,
+            rows: np.ndarray, vocab_rows: np.ndarray, block: int = 8192) -> np.ndarray:
+    """Rows `vocab_rows` of dW = G^T h, summed over the token rows `rows`:
+    dW_v = sum_t g_tv h_t with g_tv = coef_t (exp(z_tv - lse_t) - [v == x_t])
+    (the backward of Eq. 2; coef_t = m_t c_t / D and lse_t are per row, in the
+    order of `rows`).  Returns len(vocab_rows) x H, fp64."""
+    rows = np.asarray(rows)
+    vr = np.asarray(vocab_rows)
+    x_all = np.asarray(tokens)
+    Wv = W[vr]
+    out = np.zeros((vr.shape[0], hidden.shape[1]))
+    for b0 in range(0, rows.shape[0], block):
+        sl = slice(b0, min(rows.shape[0], b0 + block))
+        t = rows[sl]
+        h = hidden[t]
+        z = h @ Wv.T
+        g = np.asarray(coef)[sl][:, None] * np.exp(z - np.asarray(lse)[sl][:, None])
+        g -= np.asarray(coef)[sl][:, None] * (x_all[t][:, None] == vr[None, :])
+        out += g.T @ h
+    return out
+
+
+# --------------------------------------------------------------------------- #
+# Vocabulary-parallel pieces (the LM head split by vocabulary ranges)
+# --------------------------------------------------------------------------- #
+def shard_partials(hidden: np.ndarray, W_shard: np.ndarray, tokens: np.ndarray, v_begin: int,
+                   rows: np.ndarray):
+    """Per-row statistics of one vocabulary shard (columns v_begin ..
+    v_begin + V_shard - 1 of z = h W^T): the shard's max M_s, S_s = sum exp(z -
+    M_s), Q_s = sum exp(z - M_s)(z - M_s) and the target logit z[x] when the
+    target lies in the shard (-inf otherwise).  Returns an [n, 4] array."""
+    rows = np.asarray(rows)
+    out = np.zeros((rows.shape[0], 4))
+    Vs = W_shard.shape[0]
+    for b0 in range(0, rows.shape[0], 256):
+        sl = slice(b0, min(rows.shape[0], b0 + 256))
+        t = rows[sl]
+        z = logits_rows(hidden[t], W_shard)
+        M = z.max(axis=1)
+        e = np.exp(z - M[:, None])
+        out[sl, 0] = M
+        out[sl, 1] = e.sum(axis=1)
+        out[sl, 2] = (e * (z - M[:, None])).sum(axis=1)
+        xl = np.asarray(tokens)[t] - int(v_begin)
+        inside = (xl >= 0) & (xl < Vs)
+        zx = np.full(t.shape[0], -np.inf)
+        zx[inside] = z[np.nonzero(inside)[0], xl[inside]]
+        out[sl, 3] = zx
+    return out
+
+
+def merge_shard_partials(parts: np.ndarray):
+    """Combine the statistics of disjoint vocabulary shards ([n_shards, n, 4],
+    see shard_partials) into lse, logp and entropy of the whole row: with M the
+    largest shard max, S = sum_s S_s e^{M_s - M}, lse = M + log S, and
+    sum_v p_v z_v = sum_s e^{M_s - M} (Q_s + (M_s - M) S_s) / S + M, so that
+    entropy = lse - sum_v p_v z_v; logp = z[x] - lse from the one shard that
+    holds the target."""
+    parts = np.asarray(parts, dtype=np.float64)
+    Ms, Ss, Qs, Zs = parts[..., 0], parts[..., 1], parts[..., 2], parts[..., 3]
+    M = Ms.max(axis=0)
+    f = np.exp(Ms - M[None, :])
+    S = (Ss * f).sum(axis=0)
+    lse = M + np.log(S)
+    pz = (f * (Qs + (Ms - M[None, :]) * Ss)).sum(axis=0) / S + M
+    zx = Zs.max(axis=0)
+    return lse, zx - lse, lse - pz

@@ -400,3 +400,83 @@ def test_ex_rows_is_a_slice_of_the_full_extended_loss():
     for k in ("logp", "token_loss", "coef"):
         np.testing.assert_allclose(part[k], full[k][rows], rtol=1e-13, atol=1e-15)
     np.testing.assert_allclose(part["dH"], full["dH"][rows], rtol=1e-12, atol=1e-15)
+
+
+# ------------------------------------- full-batch forward and sampled dW rows
+def test_full_forward_rows_matches_library():
+    """lse / logp / entropy of whole rows against scipy's logsumexp,
+    log_softmax and entropy; thread splitting and row blocks change nothing;
+    large logits do not overflow (the row max is shifted out)."""
+    rng = np.random.default_rng(21)
+    T, H, V = 37, 24, 3001
+    h = rng.standard_normal((T, H))
+    W = rng.standard_normal((V, H)) * 0.5
+    x = rng.integers(0, V, T)
+    rows = np.array([36, 0, 5, 5, 17, 2])
+    z = h @ W.T
+    lse, lp, ent = O.full_forward_rows(h, W, x, rows)
+    np.testing.assert_allclose(lse, scipy.special.logsumexp(z[rows], axis=1), rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lp, scipy.special.log_softmax(z[rows], axis=1)[np.arange(6), x[rows]], atol=1e-12)
+    np.testing.assert_allclose(ent, scipy.stats.entropy(scipy.special.softmax(z[rows], axis=1), axis=1),
+                               atol=1e-12)
+    a = O.full_forward_rows(h, W, x, np.arange(T), block=7, workers=3)
+    b = O.full_forward_rows(h, W, x, np.arange(T), block=1024, workers=1)
+    for u, v in zip(a, b):
+        np.testing.assert_array_equal(u, v)
+    # a constant shift of every logit of a row moves lse by it and leaves logp
+    # and entropy alone (bias column through h)
+    h2 = np.concatenate([h, np.full((T, 1), 40.0)], axis=1)
+    W2 = np.concatenate([W, np.full((V, 1), 20.0)], axis=1)
+    lse2, lp2, ent2 = O.full_forward_rows(h2, W2, x, rows)
+    np.testing.assert_allclose(lse2, lse + 800.0, rtol=1e-14)
+    np.testing.assert_allclose(lp2, lp, atol=1e-10)
+    np.testing.assert_allclose(ent2, ent, atol=1e-9)
+
+
+def test_full_forward_rows_uniform_closed_form():
+    T, H, V = 3, 5, 777
+    lse, lp, ent = O.full_forward_rows(np.ones((T, H)), np.zeros((V, H)), np.arange(T), np.arange(T))
+    np.testing.assert_allclose(lse, math.log(V), atol=1e-13)
+    np.testing.assert_allclose(lp, -math.log(V), atol=1e-13)
+    np.testing.assert_allclose(ent, math.log(V), atol=1e-13)
+
+
+def test_dW_rows_is_a_slice_of_the_full_backward():
+    """dW_rows with the loss's own lse and m c / D reproduces rows of the full
+    backward (itself pinned by autograd and finite differences), target rows
+    (one-hot term) and non-target rows alike."""
+    h, W, x, m = _small_problem(23, T=40, H=12, V=50, mask=[1, 1, 1, 0] * 10)
+    rng = np.random.default_rng(23)
+    adv = rng.standard_normal(40)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    b = lp + rng.normal(0, 0.3, 40)
+    full = O.policy_loss(h, W, x, b, adv, m, 0.2, 0.25)
+    act = np.nonzero(m)[0]
+    vr = np.unique(np.concatenate([x[act][:5], [0, 7, 49]]))
+    got = O.dW_rows(h, W, x, full["lse"][act], full["coef"][act], act, vr, block=7)
+    np.testing.assert_allclose(got, full["dW"][vr], rtol=1e-11, atol=1e-15)
+    assert np.abs(full["dW"][vr]).max() > 0
+
+
+def test_shard_merge_equals_whole_row():
+    """Statistics of disjoint vocabulary shards merged in log space equal the
+    whole row's lse, logp and entropy, for any split (uneven shards, shards
+    without any target, one shard)."""
+    rng = np.random.default_rng(29)
+    T, H, V = 23, 16, 1000
+    h = rng.standard_normal((T, H))
+    W = rng.standard_normal((V, H)) * 0.8
+    x = rng.integers(0, 300, T)                 # targets only in the first shards
+    rows = np.arange(T)
+    ref = O.full_forward_rows(h, W, x, rows)
+    for bounds in ([0, V], [0, 500, V], [0, 1, 333, 334, V], [0, 123, 456, 789, 999, V]):
+        parts = np.stack([O.shard_partials(h, W[a:b], x, a, rows) for a, b in zip(bounds[:-1], bounds[1:])])
+        lse, lp, ent = O.merge_shard_partials(parts)
+        np.testing.assert_allclose(lse, ref[0], rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lp, ref[1], rtol=0, atol=1e-12)
+        np.testing.assert_allclose(ent, ref[2], rtol=0, atol=1e-11)
+    # a shard's own statistics: lse of the shard alone = M + log S
+    p = O.shard_partials(h, W[500:], x, 500, rows)
+    np.testing.assert_allclose(p[:, 0] + np.log(p[:, 1]), scipy.special.logsumexp((h @ W[500:].T), axis=1),
+                               atol=1e-12)
+    assert np.isneginf(p[:, 3]).all()           # no target falls in [500, V)
