@@ -11,7 +11,7 @@ in spans of 8-256, clip eps 0.2 / 0.28.  Inputs are synthetic and seeded
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--estimator grpo|group_mean|dr_grpo|rloo|reinforce_pp]
-                  [--objective ppo|kl_entropy_gate] [--deterministic]
+                  [--objective ppo|kl_entropy_gate] [--deterministic] [--vshard N]
 
 --estimator picks the advantage estimator (Sec. 4.5 list); --objective
 kl_entropy_gate adds a KL-to-reference term, an entropy bonus and the
@@ -20,6 +20,13 @@ defaults are the headline configuration (GRPO, clipped surrogate).
 
 With torchrun (N > 1) every rank processes its own batch (different seed)
 with no collective on the data path ("scaling": "weak"); rank 0 prints.
+
+--vshard N splits W by vocabulary into N shards and runs the step through the
+vocabulary-parallel calls (shard statistics, their merge with the loss, the
+shards' backward).  On one process the N shards run one after another on the
+GPU; under torchrun with N ranks, rank r holds shard r and the ranks exchange
+the statistics (all-gather) and the dhidden terms (all-reduce) over NCCL, one
+batch per step for the whole job ("scaling": "strong").
 --impl reference times the fp64 CPU oracle on the host cores instead, on a
 bounded sample of rows per step.
 """
@@ -370,6 +377,45 @@ def run_ours(args):
         return molt.policy_loss_fwd_bwd(hid, weight, tok, bb, adv_tok, msk, w.eps_lo, w.eps_hi, dW=dW,
                                         want_token_outputs=False)
 
+    vshard = args.vshard
+    mine = []
+    if vshard > 1:
+        if world not in (1, vshard):
+            raise SystemExit("--vshard N runs on one process or on N ranks")
+        if extended or args.estimator != "grpo":
+            raise SystemExit("--vshard runs the headline objective (GRPO, clipped surrogate)")
+        bounds = molt.vocab_shard_bounds(V, vshard)
+        mine = [bounds[rank]] if world > 1 else bounds
+        w_sh = [weight[a:e] for a, e in mine]
+        dW_sh = [torch.empty(e - a, H, dtype=torch.float32, device=dev) for a, e in mine]
+        dh_sum = torch.empty(T, H, dtype=torch.float32, device=dev)
+        vp_timer = {"t": None, "k": 0}
+
+        def arm():
+            if vp_timer["t"] is not None:
+                vp_timer["t"].arm(vp_timer["k"])
+                vp_timer["k"] += 1
+
+        def step(tok=tokens, msk=mask, hid=hidden, bb=b, rw=rewards, gi=gids, ro=rot, rf=None):
+            molt.group_advantages(rw, gi, out=adv_resp)
+            molt.broadcast_advantages(adv_resp, ro, out=adv_tok)
+            parts = []
+            for (a, e), ws in zip(mine, w_sh):
+                arm()
+                parts.append(molt.vp_partials(hid, ws, tok, a, msk))
+            parts = molt.gather_shard_partials(parts[0]) if world > 1 else torch.stack(parts)
+            arm()
+            out = molt.vp_loss(parts, bb, adv_tok, msk, w.eps_lo, w.eps_hi)
+            dh_sum.zero_()
+            for (a, e), ws, dws in zip(mine, w_sh, dW_sh):
+                arm()
+                dh_s, _ = molt.vp_backward(hid, ws, tok, out["lse"], out["coef"], a, dW=dws)
+                dh_sum.add_(dh_s)
+            if world > 1:
+                molt.sum_dhidden(dh_sum)
+            out["dhidden"] = dh_sum
+            return out
+
     def barrier():
         if world > 1:
             dist.barrier()
@@ -380,7 +426,10 @@ def run_ours(args):
     assert molt.device_status() == 0
     barrier()
 
-    timer = molt.KernelTimer(args.steps)
+    calls_per_step = 2 * len(mine) + 1 if vshard > 1 else 1
+    timer = molt.KernelTimer(args.steps * calls_per_step)
+    if vshard > 1:
+        vp_timer["t"] = timer
     clocks = ClockSampler(gpu_index_for(local_rank))
     clocks.start()
     time.sleep(0.3)
@@ -395,11 +444,14 @@ def run_ours(args):
     for k in range(args.steps):
         if k > 0:
             marks[k - 1].record()
-        timer.arm(k)
+        if vshard <= 1:
+            timer.arm(k)
         out = step()
     t1.record()
     launches = molt.kernel_launches() - launches0
     timer.disarm()
+    if vshard > 1:
+        vp_timer["t"] = None
     torch.cuda.synchronize()
     barrier()
     clk = clocks.stop()
@@ -417,7 +469,7 @@ def run_ours(args):
 
     # ---- end to end through the public API with host buffers
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and vshard <= 1:
         pin = lambda a: torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
         h_hid = pin(w.hidden.view(np.int16))
         h_tok, h_msk, h_b = pin(w.tokens), pin(w.mask), pin(b.cpu().numpy())
@@ -488,14 +540,19 @@ def run_ours(args):
         return 0
 
     # ---- roofline of the dominant kernel (backward): algorithmic flops = dhidden
-    # and dW products, 4 T_p H V per launch, over its CUDA-event time
-    tp = n_active
+    # and dW products, 4 T_p H V per launch, over its CUDA-event time.  T_p is
+    # the rows the backward processes (active rows with a gradient), the
+    # forward's are the active rows: rows left out never count as work done.
+    # With vocabulary shards on N ranks each rank's V is its shard's.
+    tp = step_stats["n_grad_rows"]
+    V_work = (mine[0][1] - mine[0][0]) if (vshard > 1 and world > 1) else V
     bwd_s = per["backward"] / 1e3 / args.steps
     fwd_s = per["forward"] / 1e3 / args.steps
     peak = peaks["bf16_sustained"]
-    achieved_bwd = 4.0 * tp * H * V / bwd_s / 1e12
+    achieved_bwd = 4.0 * tp * H * V_work / bwd_s / 1e12
     step_s = ms / 1e3 / args.steps
-    step_frac = 6.0 * tp * H * V / step_s / 1e12 / peak
+    step_flops = (2.0 * n_active + 4.0 * tp) * H * V_work
+    step_frac = step_flops / step_s / 1e12 / peak
     bwd_kernel = "lmhead_bwd_quad_kernel" if H % 128 == 0 else "lmhead_bwd_kernel"
     roofline = {
         "kernel": bwd_kernel, "bound": "tensor", "achieved": achieved_bwd, "peak": peak, "unit": "TFLOP/s",
@@ -511,9 +568,10 @@ def run_ours(args):
                        "can use over the last few percent of it; achieved and the event time cover both"
                        if H % 128 == 0 and not args.deterministic else None),
         "kernels_per_step": launches / args.steps,
-        "algorithmic_flops_per_launch": 4.0 * tp * H * V,
-        "executed_tflops": 6.0 * tp * H * V / bwd_s / 1e12,
-        "forward_kernel_tflops": 2.0 * tp * H * V / fwd_s / 1e12,
+        "algorithmic_flops_per_launch": 4.0 * tp * H * V_work / max(1, len(mine)),
+        "backward_rows": tp,
+        "executed_tflops": 6.0 * tp * H * V_work / bwd_s / 1e12,
+        "forward_kernel_tflops": 2.0 * n_active * H * V_work / fwd_s / 1e12,
         "kernel_ms_per_step": {k: v / args.steps for k, v in per.items()},
     }
 
@@ -528,7 +586,7 @@ def run_ours(args):
 
     line = {
         "metric": METRIC,
-        "value": job_throughput(T, world, args.steps, ms),
+        "value": job_throughput(T, 1 if vshard > 1 else world, args.steps, ms),
         "unit": "tokens/s",
         "n_gpus": world,
         "steps": args.steps,
@@ -536,17 +594,20 @@ def run_ours(args):
         "ms_per_step": ms / args.steps,
         "ms_per_step_median": ms_median,
         "higher_is_better": True,
-        "scaling": "weak",
+        "scaling": "strong" if vshard > 1 else "weak",
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic",
         "config": {"workload": workload_desc(w, microbatch_of(args)), "global_batch_tokens": world * T, "active_tokens": n_active,
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "parallelism": (f"vocab-parallel x{vshard}" + (" (shards one after another on one GPU)"
+                                                                  if world == 1 else " over NCCL")
+                                   if vshard > 1 else f"replicas x{world}" if world > 1 else "single GPU"),
+                   "backward_rows": tp,
                    "l2": l2_note(T, H, V),
-                   "active_tokens_per_s": job_throughput(n_active, world, args.steps, ms),
+                   "active_tokens_per_s": job_throughput(n_active, 1 if vshard > 1 else world, args.steps, ms),
                    "tensor_peak_frac_6THV": step_frac,
-                   "tensor_peak_frac_8THV": step_frac * 8.0 / 6.0,
-                   "tensor_peak_frac_6THV_of_burst": 6.0 * tp * H * V / step_s / 1e12 / peaks["bf16"],
+                   "tensor_peak_frac_8THV": (2.0 * n_active + 6.0 * tp) * H * V_work / step_s / 1e12 / peak,
+                   "tensor_peak_frac_6THV_of_burst": step_flops / step_s / 1e12 / peaks["bf16"],
                    "loss": loss_val, "estimator": args.estimator, "objective": args.objective,
                    "deterministic": bool(args.deterministic),
                    **({"kl_coef": 0.01, "entropy_coef": 1e-3, "gate": [0.5, 2.0],
@@ -591,6 +652,8 @@ def main():
                     help="microbatch of a windowed workload (ragged: default 1)")
     ap.add_argument("--deterministic", action="store_true",
                     help="bitwise-reproducible dW / dhidden (reduce-adds take turns in a fixed order)")
+    ap.add_argument("--vshard", type=int, default=1,
+                    help="vocabulary-parallel step over N shards (one GPU: one after another; N ranks: one each)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

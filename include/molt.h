@@ -70,6 +70,9 @@ typedef struct {
   int64_t n_active;         /* sum_i m_i */
   int64_t n_clip_low;       /* tokens on the clipped branch with A_i < 0 (rho < 1 - eps_lo) */
   int64_t n_clip_high;      /* tokens on the clipped branch with A_i > 0 (rho > 1 + eps_hi) */
+  int64_t n_grad_rows;      /* active tokens whose gradient coefficient is not 0: the rows
+                               the backward processes (masked, clipped, A = 0 and rejected
+                               rows carry no gradient and are left out) */
 } molt_stats;
 
 const char* molt_status_string(molt_status s);
@@ -231,15 +234,23 @@ molt_status molt_policy_loss_fwd_bwd(const uint16_t* hidden, const uint16_t* W, 
  *                 into dW in token-quad order and into dhidden in vocabulary
  *                 block order, each [32 x 128] slab waiting its turn on a
  *                 counter in the workspace.  The order does not depend on the
- *                 number C of clusters the backward runs (a multiple of 4; C =
- *                 36 on a GB300; the environment variable MOLT_DET_CLUSTERS
- *                 may lower it).  The C clusters wait on one another, so they
- *                 must be resident together: with other work occupying SMs for
- *                 seconds the waits time out (MOLT_DEV_TIMEOUT; nothing hangs).
- *                 Needs H % 128 == 0 (MOLT_ERR_UNSUPPORTED_SHAPE otherwise) and
- *                 the workspace of molt_policy_loss_workspace_bytes_ex (the
- *                 raster's plus the counters).  0: reduce-adds in arrival order
- *                 (results agree to fp32 rounding).
+ *                 number C of clusters of four CTAs the backward runs (see
+ *                 det_clusters).  The C clusters wait on one another, so they
+ *                 must be resident together: if other work keeps SMs busy for
+ *                 seconds, a wait gives up after about 4 s, the call's backward
+ *                 returns early with dW and dhidden incomplete, and
+ *                 molt_device_status reports MOLT_ERR_DEVICE_TIMEOUT
+ *                 (MOLT_DEV_TIMEOUT bit); nothing hangs.  Needs H % 128 == 0
+ *                 (MOLT_ERR_UNSUPPORTED_SHAPE otherwise) and the workspace of
+ *                 molt_policy_loss_workspace_bytes_ex (the raster's plus the
+ *                 counters).  0: reduce-adds in arrival order (results agree
+ *                 to fp32 rounding).
+ *   det_clusters  deterministic mode only: the number C of clusters to run, a
+ *                 multiple of 4 from 4 up to the number that fit on the device
+ *                 at once (36 on a GB300); 0 takes that maximum.  A caller that
+ *                 shares the GPU with other work can leave SMs to it with a
+ *                 smaller C.  The results are the same bits for every C.  Other
+ *                 values return MOLT_ERR_INVALID_ARG.
  */
 typedef struct {
   float kl_coef;
@@ -249,6 +260,7 @@ typedef struct {
   double gate_lo;
   double gate_hi;
   int deterministic;
+  int det_clusters;
 } molt_loss_options;
 
 /* molt_stats plus the extended objective's counters (device memory). */
@@ -279,6 +291,67 @@ molt_status molt_policy_loss_fwd_bwd_ex(const uint16_t* hidden, const uint16_t* 
                                         cudaStream_t stream);
 
 /*
+ * Vocabulary-parallel LM head (Sec. 4.1: the actor composes tensor parallelism
+ * with FSDP2, Table 2 --fsdp.tp_size).  With W split by vocabulary rows over
+ * n_shards ranks, rank r holding W_shard = W[v_begin_r, v_begin_r + V_r) with
+ * the shards covering [0, V) in order, one policy-loss step is:
+ *   1. every rank: molt_vp_partials on its shard -> partials_r [T, 4];
+ *   2. the caller gathers them in shard order into partials [n_shards, T, 4]
+ *      (an all-gather of 16 bytes per token);
+ *   3. every rank: molt_vp_loss on the gathered statistics -> the loss of
+ *      Eq. 2, lse and m c / D per token (identical on every rank);
+ *   4. every rank: molt_vp_backward on its shard -> its dW shard and its
+ *      contribution to dhidden; the caller sums the contributions over the
+ *      ranks (an all-reduce of T x H fp32).
+ * The library performs no collective; the exchange of steps 2 and 4 is the
+ * caller's (NCCL, or any other transport).  Results agree with
+ * molt_policy_loss_fwd_bwd on the whole W to fp32 rounding.
+ */
+
+/* Per-token statistics of one vocabulary shard:
+ *   partials_out[t] = (M, S, Q, z_x) fp32, 16-byte aligned [T, 4], with z the
+ *   logits of the shard's columns, M = max z, S = sum exp(z - M),
+ *   Q = sum exp(z - M) (z - M), and z_x the logit of tokens[t] if it lies in
+ *   [v_begin, v_begin + V_shard), else -inf.  Rows with mask 0 (mask may be
+ *   NULL) get (-inf, 0, 0, -inf).
+ * hidden [T,H] bf16, W_shard [V_shard,H] bf16, tokens [T] int32 (global ids).
+ * Workspace as molt_token_logprobs_fwd (NULL allocates stream-ordered). */
+size_t molt_vp_partials_workspace_bytes(int64_t T, int64_t H, int64_t V_shard);
+molt_status molt_vp_partials(const uint16_t* hidden, const uint16_t* W_shard, const int32_t* tokens,
+                             const uint8_t* mask, int64_t T, int64_t H, int64_t V_shard, int64_t v_begin,
+                             float* partials_out, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* Merge of the shards' statistics (partials [n_shards, T, 4], shard order,
+ * 16-byte aligned) into each active row's lse = M + log S (M the largest
+ * shard max, S = sum_s S_s exp(M_s - M)), logp = z_x - lse and entropy, then
+ * the clipped surrogate and Eq. 2 exactly as molt_policy_loss_fwd_bwd's
+ * forward half: loss_out (device fp32 scalar), lse_out [T] and coef_out [T]
+ * (= m c / D, the inputs of molt_vp_backward; 0 on masked and clipped rows),
+ * optional logp_out, entropy_out, token_loss_out [T] and stats_out (its
+ * n_grad_rows counts the rows with coef != 0).  The reductions run in a fixed
+ * order, so every rank that merges the same statistics gets the same bits.  A
+ * row whose token lies in no shard sets MOLT_DEV_TOKEN_RANGE. */
+size_t molt_vp_loss_workspace_bytes(int64_t T);
+molt_status molt_vp_loss(const float* partials, int n_shards, const float* behavior_logp, const float* adv,
+                         const uint8_t* mask, int64_t T, float clip_lo, float clip_hi, double denom, float* loss_out,
+                         float* lse_out, float* coef_out, float* logp_out, float* entropy_out, float* token_loss_out,
+                         molt_stats* stats_out, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/* Backward of one shard: with g_tv = coef[t] (softmax(z_t)_v - [v == tokens[t]])
+ * over the shard's columns (lse and coef from molt_vp_loss),
+ *   dhidden_partial_out [T,H] fp32 = g W_shard (this shard's term of dhidden;
+ *                                    rows with coef 0 are exactly 0)
+ *   dW_shard_out [V_shard,H] fp32 (+)= g^T hidden (accumulate_dW as in
+ *                                    molt_policy_loss_fwd_bwd).
+ * Only rows with coef != 0 are computed.  16-byte-aligned outputs.  The
+ * workspace holds the packed rows and an fp32 [T,H] accumulator. */
+size_t molt_vp_backward_workspace_bytes(int64_t T, int64_t H, int64_t V_shard);
+molt_status molt_vp_backward(const uint16_t* hidden, const uint16_t* W_shard, const int32_t* tokens,
+                             const float* lse, const float* coef, int64_t T, int64_t H, int64_t V_shard,
+                             int64_t v_begin, float* dhidden_partial_out, float* dW_shard_out, int accumulate_dW,
+                             void* workspace, size_t workspace_bytes, cudaStream_t stream);
+
+/*
  * Allocation-free variant of molt_token_logprobs_fwd (the paper has no
  * counterpart; it exists for callers, not for the method).
  *
@@ -299,7 +372,10 @@ molt_status molt_policy_loss_fwd_bwd_ex(const uint16_t* hidden, const uint16_t* 
  *     them, e.g. by issuing them on one stream.
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress, with that device current); later calls reuse it.
+ *     A lookup that fails is not remembered: the next call tries again.
  *     Make the first call on a device before any stream capture on it.
+ *   - The timing hook (molt_set_timing_events) records kernel groups 1 (the
+ *     forward kernel) and 2 (the merge) of this call.
  * Masked rows are computed and then written as 0 (there is no compaction),
  * so prefer molt_token_logprobs_fwd when allocation is allowed.
  */
@@ -314,7 +390,8 @@ molt_status molt_token_logprobs_fwd_noalloc(const uint16_t* hidden, const uint16
  * events) on its stream around kernel group k:
  *   k = 0  active-row compaction and packed gather
  *   k = 1  LM-head forward kernel (online log-softmax)
- *   k = 2  split merge, surrogate loss and the fixed-order reductions
+ *   k = 2  split merge, surrogate loss, the fixed-order reductions and the
+ *          packing of the rows with a gradient for the backward
  *   k = 3  LM-head backward kernel (dhidden / dW products)
  *   k = 4  dhidden cast
  * Slots beyond n are ignored.  n = 0 (or NULL arrays) turns the hook off.

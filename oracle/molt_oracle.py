@@ -66,7 +66,7 @@ __all__ = [
     "widen_bf16", "group_advantages", "advantages", "ESTIMATORS", "broadcast_advantages", "logits_rows",
     "row_softmax_stats", "token_logprobs", "policy_loss", "policy_loss_rows",
     "clip_decision", "surrogate", "policy_loss_ex", "sequence_gate", "policy_loss_ex_rows",
-    "full_forward_rows", "dW_rows", "shard_partials", "merge_shard_partials",
+    "full_forward_rows", "dW_rows", "shard_partials", "merge_shard_partials", "shard_dhidden",
 ]
 
 DEFAULT_ADV_EPS = 1e-6
@@ -593,3 +593,25 @@ def merge_shard_partials(parts: np.ndarray):
     pz = (f * (Qs + (Ms - M[None, :]) * Ss)).sum(axis=0) / S + M
     zx = Zs.max(axis=0)
     return lse, zx - lse, lse - pz
+
+
+def shard_dhidden(hidden: np.ndarray, W_shard: np.ndarray, tokens: np.ndarray, v_begin: int, lse: np.ndarray,
+                  coef: np.ndarray, rows: np.ndarray) -> np.ndarray:
+    """One vocabulary shard's term of dhidden for the given rows:
+    sum over the shard's columns v of g_tv W_v, with g_tv = coef_t
+    (exp(z_tv - lse_t) - [v == x_t]) and lse_t, coef_t of the whole row (in
+    the order of `rows`).  The shards' terms sum to dH = G W."""
+    rows = np.asarray(rows)
+    Vs = W_shard.shape[0]
+    out = np.zeros((rows.shape[0], hidden.shape[1]))
+    for b0 in range(0, rows.shape[0], 256):
+        sl = slice(b0, min(rows.shape[0], b0 + 256))
+        t = rows[sl]
+        z = logits_rows(hidden[t], W_shard)
+        c = np.asarray(coef)[sl]
+        g = c[:, None] * np.exp(z - np.asarray(lse)[sl][:, None])
+        xl = np.asarray(tokens)[t] - int(v_begin)
+        inside = np.nonzero((xl >= 0) & (xl < Vs))[0]
+        g[inside, xl[inside]] -= c[inside]
+        out[sl] = g @ W_shard
+    return out

@@ -20,6 +20,8 @@ __all__ = [
     "build", "load", "lib_path", "MoltError", "STATUS", "DEV_FLAGS", "group_advantages",
     "broadcast_advantages", "mask_count", "token_logprobs", "policy_loss_fwd_bwd", "device_status",
     "token_logprobs_workspace_bytes", "policy_loss_workspace_bytes", "header_functions",
+    "vp_partials", "vp_loss", "vp_backward", "vocab_shard_bounds", "gather_shard_partials", "sum_dhidden",
+    "policy_loss_vocab_parallel",
 ]
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
@@ -125,6 +127,12 @@ def load():
                                                P, P, P, SZ, P]),
         "molt_set_timing_events": (None, [P, P, I32]),
         "molt_token_logprobs_fwd_noalloc": (I32, [P, P, P, P, I64, I64, I64, P, P, P]),
+        "molt_vp_partials_workspace_bytes": (SZ, [I64, I64, I64]),
+        "molt_vp_partials": (I32, [P, P, P, P, I64, I64, I64, I64, P, P, SZ, P]),
+        "molt_vp_loss_workspace_bytes": (SZ, [I64]),
+        "molt_vp_loss": (I32, [P, I32, P, P, P, I64, F, F, D, P, P, P, P, P, P, P, P, SZ, P]),
+        "molt_vp_backward_workspace_bytes": (SZ, [I64, I64, I64]),
+        "molt_vp_backward": (I32, [P, P, P, P, P, I64, I64, I64, I64, P, P, I32, P, SZ, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -354,12 +362,22 @@ def token_logprobs(hidden, weight, tokens, mask=None, want_entropy=True, stream=
     return logp, ent
 
 
-NOALLOC_MAX_TOKENS = 32768
+def _header_define(name: str) -> int:
+    with open(os.path.join(_INCLUDE, "molt.h")) as f:
+        m = re.search(r"#define\s+" + name + r"\s+(\d+)", f.read())
+    if m is None:
+        raise RuntimeError(f"{name} is not defined in molt.h")
+    return int(m.group(1))
+
+
+# the largest T molt_token_logprobs_fwd_noalloc takes (MOLT_NOALLOC_MAX_TOKENS)
+NOALLOC_MAX_TOKENS = _header_define("MOLT_NOALLOC_MAX_TOKENS")
 
 
 def token_logprobs_noalloc(hidden, weight, tokens, mask=None, want_entropy=True, stream=None):
     """Like token_logprobs, through molt_token_logprobs_fwd_noalloc: the library
-    allocates nothing (its scratch is a fixed device array); T <= 32768."""
+    allocates nothing (its scratch is a fixed device array); T is at most
+    NOALLOC_MAX_TOKENS."""
     torch = _torch()
     T, H = hidden.shape
     V = weight.shape[0]
@@ -378,7 +396,7 @@ def policy_loss_fwd_bwd(hidden, weight, tokens, behavior_logp, adv, mask=None, c
     """Fused clipped-surrogate loss (Eq. 2 token-mean) forward + backward.
 
     Returns dict(loss [1] fp32, dhidden [T,H] bf16, dW [V,H] fp32, logp, entropy,
-    token_loss [T] fp32 (None unless want_token_outputs), stats [8 x 8 bytes])."""
+    token_loss [T] fp32 (None unless want_token_outputs), stats [9 x 8 bytes])."""
     torch = _torch()
     T, H = hidden.shape
     V = weight.shape[0]
@@ -388,7 +406,7 @@ def policy_loss_fwd_bwd(hidden, weight, tokens, behavior_logp, adv, mask=None, c
     if dW is None:
         dW = torch.empty(V, H, dtype=torch.float32, device=dev)
         accumulate_dW = False
-    stats = torch.zeros(8, dtype=torch.float64, device=dev)
+    stats = torch.zeros(9, dtype=torch.float64, device=dev)
     logp = ent = tl = None
     if want_token_outputs:
         logp = torch.empty(T, dtype=torch.float32, device=dev)
@@ -407,18 +425,18 @@ def policy_loss_fwd_bwd(hidden, weight, tokens, behavior_logp, adv, mask=None, c
 
 
 def stats_dict(stats_tensor) -> dict:
-    """Decode molt_stats (5 doubles + 3 int64) or molt_stats_ex (those, then
+    """Decode molt_stats (5 doubles + 4 int64) or molt_stats_ex (those, then
     1 double + 2 int64) copied to the host."""
     import numpy as np
     raw = stats_tensor.detach().cpu().numpy().view(np.uint8).tobytes()
     d = np.frombuffer(raw[:40], dtype=np.float64)
-    i = np.frombuffer(raw[40:64], dtype=np.int64)
+    i = np.frombuffer(raw[40:72], dtype=np.int64)
     out = {"denom": float(d[0]), "loss": float(d[1]), "sum_ratio": float(d[2]), "sum_entropy": float(d[3]),
            "max_abs_log_ratio": float(d[4]), "n_active": int(i[0]), "n_clip_low": int(i[1]),
-           "n_clip_high": int(i[2])}
-    if len(raw) >= 88:
-        out["sum_kl"] = float(np.frombuffer(raw[64:72], dtype=np.float64)[0])
-        j = np.frombuffer(raw[72:88], dtype=np.int64)
+           "n_clip_high": int(i[2]), "n_grad_rows": int(i[3])}
+    if len(raw) >= 96:
+        out["sum_kl"] = float(np.frombuffer(raw[72:80], dtype=np.float64)[0])
+        j = np.frombuffer(raw[80:96], dtype=np.int64)
         out["n_tokens_rejected"] = int(j[0])
         out["n_seq_rejected"] = int(j[1])
     return out
@@ -428,16 +446,18 @@ class LossOptions(ctypes.Structure):
     """molt_loss_options: KL-to-reference, entropy bonus, sequence gate."""
     _fields_ = [("kl_coef", ctypes.c_float), ("entropy_coef", ctypes.c_float), ("ref_logp", ctypes.c_void_p),
                 ("seq_of_token", ctypes.c_void_p), ("gate_lo", ctypes.c_double), ("gate_hi", ctypes.c_double),
-                ("deterministic", ctypes.c_int)]
+                ("deterministic", ctypes.c_int), ("det_clusters", ctypes.c_int)]
 
 
 def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None, clip_lo=0.2, clip_hi=0.2,
                            denom=0.0, kl_coef=0.0, ref_logp=None, entropy_coef=0.0, seq_of_token=None,
-                           gate_lo=0.0, gate_hi=float("inf"), deterministic=False, dW=None, accumulate_dW=False,
-                           want_token_outputs=True, stream=None, workspace=None):
+                           gate_lo=0.0, gate_hi=float("inf"), deterministic=False, det_clusters=0, dW=None,
+                           accumulate_dW=False, want_token_outputs=True, stream=None, workspace=None):
     """policy_loss_fwd_bwd with the extended objective
     l_t = w_t (l_pg,t + kl_coef KL_t - entropy_coef H_t) (molt_policy_loss_fwd_bwd_ex).
-    Returns the same dict; stats is molt_stats_ex (11 x 8 bytes)."""
+    det_clusters (deterministic mode): clusters of four CTAs to run, a multiple
+    of 4, or 0 for all that fit; the results do not depend on it.
+    Returns the same dict; stats is molt_stats_ex (12 x 8 bytes)."""
     torch = _torch()
     T, H = hidden.shape
     V = weight.shape[0]
@@ -447,7 +467,7 @@ def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None
     if dW is None:
         dW = torch.empty(V, H, dtype=torch.float32, device=dev)
         accumulate_dW = False
-    stats = torch.zeros(11, dtype=torch.float64, device=dev)
+    stats = torch.zeros(12, dtype=torch.float64, device=dev)
     logp = ent = tl = None
     if want_token_outputs:
         logp = torch.empty(T, dtype=torch.float32, device=dev)
@@ -455,7 +475,7 @@ def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None
         tl = torch.empty(T, dtype=torch.float32, device=dev)
     opts = LossOptions(float(kl_coef), float(entropy_coef), _ptr(ref_logp, torch.float32, "ref_logp"),
                        _ptr(seq_of_token, torch.int32, "seq_of_token"), float(gate_lo), float(gate_hi),
-                       1 if deterministic else 0)
+                       1 if deterministic else 0, int(det_clusters))
     nbytes = int(load().molt_policy_loss_workspace_bytes_ex(T, H, V, ctypes.byref(opts)))
     if nbytes == 0:
         raise MoltError(2, "unsupported shape for these options")
@@ -468,3 +488,107 @@ def policy_loss_fwd_bwd_ex(hidden, weight, tokens, behavior_logp, adv, mask=None
         _ptr(logp), _ptr(ent), _ptr(tl), _ptr(stats), ws.data_ptr(), ws.numel(), _stream(stream)))
     return {"loss": loss, "dhidden": dh, "dW": dW, "logp": logp, "entropy": ent, "token_loss": tl,
             "stats": stats}
+
+
+# ------------------------------------------------------- vocabulary parallel
+def vocab_shard_bounds(V: int, n_shards: int) -> list:
+    """[(v_begin, v_end)] of n_shards contiguous vocabulary ranges covering
+    [0, V) in order (rank r holds the r-th)."""
+    if n_shards < 1 or n_shards > V:
+        raise ValueError("need 1 <= n_shards <= V")
+    return [(r * V // n_shards, (r + 1) * V // n_shards) for r in range(n_shards)]
+
+
+def vp_partials(hidden, weight_shard, tokens, v_begin, mask=None, stream=None, workspace=None):
+    """Per-token statistics (M, S, Q, z_x) of one vocabulary shard
+    (molt_vp_partials): fp32 [T, 4]."""
+    torch = _torch()
+    T, H = hidden.shape
+    Vs = weight_shard.shape[0]
+    out = torch.empty(T, 4, dtype=torch.float32, device=hidden.device)
+    nbytes = int(load().molt_vp_partials_workspace_bytes(T, H, Vs))
+    ws = workspace if workspace is not None else _workspace(nbytes, hidden.device, "logprobs", stream)
+    _check(load().molt_vp_partials(_bf16_bits(hidden, "hidden"), _bf16_bits(weight_shard, "weight_shard"),
+                                   _ptr(tokens, torch.int32, "tokens"), _ptr(mask, torch.uint8, "mask"), T, H, Vs,
+                                   int(v_begin), _ptr(out), ws.data_ptr(), ws.numel(), _stream(stream)))
+    return out
+
+
+def vp_loss(partials, behavior_logp, adv, mask=None, clip_lo=0.2, clip_hi=0.2, denom=0.0, stream=None):
+    """Merge of the shards' statistics ([n_shards, T, 4], shard order) with
+    the clipped surrogate and Eq. 2 (molt_vp_loss).  Returns dict(loss, lse,
+    coef, logp, entropy, token_loss, stats)."""
+    torch = _torch()
+    n, T, four = partials.shape
+    if four != 4:
+        raise ValueError("partials must be [n_shards, T, 4]")
+    dev = partials.device
+    out = {"loss": torch.empty(1, dtype=torch.float32, device=dev)}
+    for k in ("lse", "coef", "logp", "entropy", "token_loss"):
+        out[k] = torch.empty(T, dtype=torch.float32, device=dev)
+    out["stats"] = torch.zeros(9, dtype=torch.float64, device=dev)
+    nbytes = int(load().molt_vp_loss_workspace_bytes(T))
+    ws = _workspace(nbytes, dev, "vp_loss", stream)
+    _check(load().molt_vp_loss(
+        _ptr(partials, torch.float32, "partials"), n, _ptr(behavior_logp, torch.float32, "behavior_logp"),
+        _ptr(adv, torch.float32, "adv"), _ptr(mask, torch.uint8, "mask"), T, float(clip_lo), float(clip_hi),
+        float(denom), _ptr(out["loss"]), _ptr(out["lse"]), _ptr(out["coef"]), _ptr(out["logp"]),
+        _ptr(out["entropy"]), _ptr(out["token_loss"]), _ptr(out["stats"]), ws.data_ptr(), ws.numel(),
+        _stream(stream)))
+    return out
+
+
+def vp_backward(hidden, weight_shard, tokens, lse, coef, v_begin, dW=None, accumulate_dW=False, stream=None):
+    """One shard's backward (molt_vp_backward): returns (dhidden contribution
+    fp32 [T, H], dW shard fp32 [V_shard, H])."""
+    torch = _torch()
+    T, H = hidden.shape
+    Vs = weight_shard.shape[0]
+    dev = hidden.device
+    dh = torch.empty(T, H, dtype=torch.float32, device=dev)
+    if dW is None:
+        dW = torch.empty(Vs, H, dtype=torch.float32, device=dev)
+        accumulate_dW = False
+    nbytes = int(load().molt_vp_backward_workspace_bytes(T, H, Vs))
+    ws = _workspace(nbytes, dev, "vp_backward", stream)
+    _check(load().molt_vp_backward(
+        _bf16_bits(hidden, "hidden"), _bf16_bits(weight_shard, "weight_shard"), _ptr(tokens, torch.int32, "tokens"),
+        _ptr(lse, torch.float32, "lse"), _ptr(coef, torch.float32, "coef"), T, H, Vs, int(v_begin), _ptr(dh),
+        _ptr(dW, torch.float32, "dW"), 1 if accumulate_dW else 0, ws.data_ptr(), ws.numel(), _stream(stream)))
+    return dh, dW
+
+
+def gather_shard_partials(local, group=None):
+    """The exchange before the merge: every rank's [T, 4] statistics, stacked
+    in rank order (rank r holds the r-th vocabulary range) -> [n_shards, T, 4].
+    One all-gather of 16 bytes per token over torch.distributed."""
+    torch = _torch()
+    import torch.distributed as dist
+    world = dist.get_world_size(group)
+    bufs = [torch.empty_like(local) for _ in range(world)]
+    dist.all_gather(bufs, local.contiguous(), group=group)
+    return torch.stack(bufs)
+
+
+def sum_dhidden(partial, group=None):
+    """The exchange after the shards' backward: dhidden = the sum of every
+    rank's contribution (all-reduce, in place)."""
+    import torch.distributed as dist
+    dist.all_reduce(partial, op=dist.ReduceOp.SUM, group=group)
+    return partial
+
+
+def policy_loss_vocab_parallel(hidden, weight_shard, v_begin, tokens, behavior_logp, adv, mask=None, clip_lo=0.2,
+                               clip_hi=0.2, denom=0.0, group=None, stream=None):
+    """One rank's policy-loss step with W split by vocabulary over the ranks
+    of `group` (rank r holds W[v_begin_r : v_begin_r + V_r], in order):
+    shard statistics -> all-gather -> merge and loss -> shard backward ->
+    all-reduce of dhidden.  Returns the vp_loss dict plus dhidden (fp32, the
+    sum over the ranks) and dW (this rank's shard)."""
+    local = vp_partials(hidden, weight_shard, tokens, v_begin, mask, stream=stream)
+    parts = gather_shard_partials(local, group)
+    out = vp_loss(parts, behavior_logp, adv, mask, clip_lo, clip_hi, denom, stream=stream)
+    dh, dW = vp_backward(hidden, weight_shard, tokens, out["lse"], out["coef"], v_begin, stream=stream)
+    out["dhidden"] = sum_dhidden(dh, group)
+    out["dW"] = dW
+    return out

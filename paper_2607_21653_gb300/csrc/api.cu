@@ -2,7 +2,6 @@
 // layout, TMA tensor maps and the launch sequence of each entry point.
 #include <atomic>
 #include <cstdint>
-#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -131,7 +130,8 @@ int choose_splits(int64_t Tcap, int64_t V, int n_sm) {
 
 struct Layout {
   size_t counts, row_map, pos, tok_p, b_p, adv_p, h_p, part, zx, lse, coef, tile_flag, tile_list, red, dh32, turns;
-  size_t lp_p, ent_p, ecoef, mu, gate_p, total;
+  size_t lp_p, ent_p, ecoef, mu, gate_p;
+  size_t live_map, live_of, h_l, tok_l, lse_l, coef_l, ecoef_l, mu_l, total;
 };
 
 constexpr size_t kNoRegion = ~size_t(0);   // a Layout region that is not allocated
@@ -184,7 +184,72 @@ Layout layout(int64_t T, int64_t H, int64_t V, int S, bool with_bwd, bool det = 
   L.ecoef = with_bwd ? take(Tcap * 4) : o;
   L.mu = with_bwd ? take(Tcap * 4) : o;
   L.gate_p = with_bwd ? take(Tcap) : o;
+  L.live_map = with_bwd ? take(Tcap * 4) : o;
+  L.live_of = with_bwd ? take(Tcap * 4) : o;
+  L.h_l = with_bwd ? take(Tcap * H * 2) : o;
+  L.tok_l = with_bwd ? take(Tcap * 4) : o;
+  L.lse_l = with_bwd ? take(Tcap * 4) : o;
+  L.coef_l = with_bwd ? take(Tcap * 4) : o;
+  L.ecoef_l = with_bwd ? take(Tcap * 4) : o;
+  L.mu_l = with_bwd ? take(Tcap * 4) : o;
   L.total = o + 256;   // slack for aligning the caller's base pointer
+  return L;
+}
+
+// Workspace of the shard merge (molt_vp_loss): the active-row compaction,
+// per-row m c / D, the tile partial sums and finalize's row list.
+Layout vp_loss_layout(int64_t T) {
+  const int64_t Tcap = round_tiles(T);
+  const int64_t ntile = Tcap / kTileM;
+  Layout L{};
+  size_t o = 0;
+  auto take = [&o](size_t bytes) {
+    size_t r = o;
+    o += up256(bytes);
+    return r;
+  };
+  L.counts = take(64);
+  L.row_map = take(T * 4);
+  L.pos = take(T * 4);
+  L.coef = take(Tcap * 4);
+  L.tile_flag = take(ntile * 4);
+  L.tile_list = take(ntile * 4);
+  L.red = take(ntile * kRedSlots * 8);
+  L.live_map = take(Tcap * 4);
+  L.live_of = take(Tcap * 4);
+  L.tok_p = L.b_p = L.adv_p = L.h_p = L.part = L.zx = L.lse = L.dh32 = L.lp_p = L.ent_p = L.ecoef = L.mu = L.gate_p =
+      L.h_l = L.tok_l = L.lse_l = L.coef_l = L.ecoef_l = L.mu_l = o;
+  L.turns = kNoRegion;
+  L.total = o + 256;
+  return L;
+}
+
+// Workspace of one shard's backward (molt_vp_backward): the rows with a
+// gradient, packed (hidden, token, lse, m c / D), and the fp32 dhidden
+// accumulator by backward row.
+Layout vp_backward_layout(int64_t T, int64_t H) {
+  const int64_t Tcap = round_tiles(T);
+  const int64_t ntile = Tcap / kTileM;
+  Layout L{};
+  size_t o = 0;
+  auto take = [&o](size_t bytes) {
+    size_t r = o;
+    o += up256(bytes);
+    return r;
+  };
+  L.counts = take(64);
+  L.tile_list = take(ntile * 4);
+  L.live_map = take(Tcap * 4);
+  L.live_of = take(Tcap * 4);
+  L.h_l = take(Tcap * H * 2);
+  L.tok_l = take(Tcap * 4);
+  L.lse_l = take(Tcap * 4);
+  L.coef_l = take(Tcap * 4);
+  L.dh32 = take(static_cast<size_t>(Tcap) * H * 4);
+  L.row_map = L.pos = L.tok_p = L.b_p = L.adv_p = L.h_p = L.part = L.zx = L.lse = L.coef = L.tile_flag = L.red =
+      L.lp_p = L.ent_p = L.ecoef = L.mu = L.gate_p = L.ecoef_l = L.mu_l = o;
+  L.turns = kNoRegion;
+  L.total = o + 256;
   return L;
 }
 
@@ -212,6 +277,14 @@ Workspace carve(void* base, const Layout& L) {
   w.ecoef = reinterpret_cast<float*>(p + L.ecoef);
   w.mu = reinterpret_cast<float*>(p + L.mu);
   w.gate_p = p + L.gate_p;
+  w.live_map = reinterpret_cast<int32_t*>(p + L.live_map);
+  w.live_of = reinterpret_cast<int32_t*>(p + L.live_of);
+  w.h_l = reinterpret_cast<uint16_t*>(p + L.h_l);
+  w.tok_l = reinterpret_cast<int32_t*>(p + L.tok_l);
+  w.lse_l = reinterpret_cast<float*>(p + L.lse_l);
+  w.coef_l = reinterpret_cast<float*>(p + L.coef_l);
+  w.ecoef_l = reinterpret_cast<float*>(p + L.ecoef_l);
+  w.mu_l = reinterpret_cast<float*>(p + L.mu_l);
   return w;
 }
 
@@ -356,14 +429,16 @@ const SideLane* side_lane(cudaStream_t caller) {
 
 // Shared front half of both LM-head calls: compaction, packed gather and the
 // forward kernel (tensor maps already encoded by the caller).
+// tok_shift is subtracted from the tokens (a vocabulary shard's first column).
 molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int32_t* tokens, const uint8_t* mask,
                         const float* b, const float* adv, int64_t T, int64_t H, int64_t V, int S,
-                        const Workspace& w, const CUtensorMap& tm_h, const CUtensorMap& tm_w, cudaStream_t s) {
+                        const Workspace& w, const CUtensorMap& tm_h, const CUtensorMap& tm_w, cudaStream_t s,
+                        int tok_shift = 0) {
   const int64_t Tcap = round_tiles(T);
   ev_start(0, s);
   MOLT_LAUNCH(launch_compact(mask, static_cast<int>(T), w, s), "compact");
   MOLT_LAUNCH(launch_gather(hidden, tokens, b, adv, static_cast<int>(T), static_cast<int>(Tcap), static_cast<int>(H),
-                          w, di->n_sm, s),
+                          w, di->n_sm, s, tok_shift),
             "gather");
   ev_stop(0, s);
   FwdArgs fa{};
@@ -380,6 +455,105 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
   ev_start(1, s);
   MOLT_LAUNCH(launch_lmhead_fwd(tm_h, tm_w, fa, di->n_sm, s), "lmhead forward");
   ev_stop(1, s);
+  return MOLT_OK;
+}
+
+// Back half of the loss calls: the backward kernels over the rows with a
+// gradient, packed in w (h_l, tok_l, lse_l, coef_l and, with an entropy bonus,
+// ecoef_l and mu_l; counts[1] tiles of them), reduce-adding into the fp32
+// accumulator w.dh32 (by backward row) and dW (zeroed first unless
+// accumulate_dW).  det: the deterministic schedule on n_det clusters.
+molt_status run_backward(const DeviceInfo* di, const uint16_t* W, int64_t T, int64_t H, int64_t V,
+                         const Workspace& w, bool det, int n_det, bool with_ecoef, float* dW_out, int accumulate_dW,
+                         cudaStream_t stream) {
+  const int64_t Tcap = round_tiles(T);
+  const bool pair_bwd = (H % 128) == 0;   // the cluster backward
+  CUtensorMap tm_wz, tm_wn, tm_dh, tm_dw;
+  MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, pair_bwd ? 128 : kBwdBV));
+  MOLT_TRY(make_tmap(&tm_wn, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, 64));
+  // the backward reads the rows with a gradient, packed again into h_l:
+  // 128-row boxes for the single-CTA kernel, 64-byte-swizzled K = 32 boxes of
+  // h and W for the logit recompute on CTA pairs, and 64-row boxes of h (a dW
+  // stage of the cluster backward is 64 token rows)
+  CUtensorMap tm_hb, tm_hz, tm_wz32, tm_h64;
+  MOLT_TRY(make_tmap(&tm_hb, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_l, Tcap, H, kBK, kTileM));
+  MOLT_TRY(make_tmap(&tm_hz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_l, Tcap, H, 32, kTileM,
+                     CU_TENSOR_MAP_SWIZZLE_64B));
+  MOLT_TRY(make_tmap(&tm_wz32, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, 32, 128, CU_TENSOR_MAP_SWIZZLE_64B));
+  MOLT_TRY(make_tmap(&tm_h64, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_l, Tcap, H, kBK, 64));
+  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
+  MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
+  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
+  const TurnLayout tl = turn_layout(Tcap, H, V);
+  if (det) MOLT_CUDA(cudaMemsetAsync(w.turns, 0, static_cast<size_t>(tl.words) * 4, stream), "memset turns");
+  if (!accumulate_dW)
+    MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
+  BwdArgs ba{};
+  ba.tok_p = w.tok_l;
+  ba.lse = w.lse_l;
+  ba.coef = w.coef_l;
+  ba.counts = w.counts;
+  ba.tile_list = w.tile_list;
+  ba.V = static_cast<int>(V);
+  ba.H = static_cast<int>(H);
+  ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
+  ba.tile_group = pair_bwd ? 4 : 16;
+  ba.dh32 = w.dh32;
+  ba.dW = dW_out;
+  ba.det_clusters = n_det;
+  if (det) {
+    ba.det_abort = w.turns;
+    ba.det_dh_turns = w.turns + tl.dh_off;
+    ba.det_dw_turns = w.turns + tl.dw_off;
+  }
+  if (with_ecoef) {
+    ba.ecoef = w.ecoef_l;
+    ba.mu = w.mu_l;
+  }
+  ba.err = di->status;
+  ev_start(3, stream);
+  if (pair_bwd) {
+    // vocab split with the single-CTA kernel on the SMs no cluster can use
+    // (raster schedule only: the deterministic order needs every vocab block
+    // reduced by its owner clusters)
+    const int clusters = lmhead_bwd_quad_clusters(di->n_sm);
+    const int spare = di->n_sm - 4 * clusters;
+    int64_t Vq = V;
+    const SideLane* lane = nullptr;
+    if (!det) {
+      const int64_t vq = choose_vocab_split(T, V, clusters, spare);
+      if (vq < V && (lane = side_lane(stream)) != nullptr) Vq = vq;
+    }
+    if (Vq < V) {
+      CUtensorMap tm_wz256;
+      MOLT_TRY(make_tmap(&tm_wz256, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kBwdBV));
+      BwdArgs bq = ba;
+      bq.V = static_cast<int>(Vq);   // columns from Vq on count as padding for the cluster kernel
+      BwdArgs bs = ba;
+      bs.vc_begin = static_cast<int>(Vq / kBwdBV);
+      bs.n_vchunks = static_cast<int>((V - Vq + kBwdBV - 1) / kBwdBV);
+      bs.tile_group = 16;
+      // the cluster kernel is enqueued first so that its clusters take their
+      // SMs before the side kernel's CTAs fill the rest
+      MOLT_CUDA(cudaEventRecord(lane->fork, stream), "backward fork");
+      MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, bq, di->n_sm, stream),
+                "lmhead backward");
+      MOLT_CUDA(cudaStreamWaitEvent(lane->side, lane->fork, 0), "backward fork");
+      // the join is made whatever the side launch returned, so that nothing on
+      // the caller's stream (the workspace release included) can overtake it
+      const cudaError_t e_side = launch_lmhead_bwd(tm_hb, tm_wz256, tm_wn, tm_dh, tm_dw, bs, spare, lane->side);
+      if (e_side == cudaSuccess) note_launches(1);
+      cudaError_t e_join = cudaEventRecord(lane->join, lane->side);
+      if (e_join == cudaSuccess) e_join = cudaStreamWaitEvent(stream, lane->join, 0);
+      if (e_side != cudaSuccess) return cuda_fail(e_side, "lmhead backward (side)");
+      if (e_join != cudaSuccess) return cuda_fail(e_join, "backward join");
+    } else {
+      MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
+                "lmhead backward");
+    }
+  } else
+    MOLT_LAUNCH(launch_lmhead_bwd(tm_hb, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
+  ev_stop(3, stream);
   return MOLT_OK;
 }
 
@@ -436,33 +610,21 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   // once, whose reduce-adds take turns
   int n_det = det ? lmhead_bwd_quad_det_clusters(di->n_sm) : 0;
   if (det && n_det < 4) return fail(MOLT_ERR_UNSUPPORTED_SHAPE, "deterministic mode needs 4 clusters of 4 CTAs");
-  if (det) {
-    // MOLT_DET_CLUSTERS: fewer clusters (a multiple of 4); the results do not
-    // depend on the count
-    const char* env = std::getenv("MOLT_DET_CLUSTERS");
-    const int want = env ? std::atoi(env) : 0;
-    if (want >= 4 && want % 4 == 0 && want < n_det) n_det = want;
+  if (det && opts->det_clusters != 0) {
+    // fewer clusters (a multiple of 4); the results do not depend on the count
+    const int want = opts->det_clusters;
+    if (want < 4 || want % 4 != 0 || want > n_det)
+      return fail(MOLT_ERR_INVALID_ARG,
+                  "det_clusters must be 0 or a multiple of 4 from 4 to " + std::to_string(n_det));
+    n_det = want;
   }
   const Layout L = layout(T, H, V, S, true, det);
   Scratch sc;
   MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
   const Workspace w = carve(sc.ptr, L);
-  const bool pair_bwd = (H % 128) == 0;   // the cluster backward
-  CUtensorMap tm_h, tm_w, tm_wz, tm_wn, tm_dh, tm_dw;
+  CUtensorMap tm_h, tm_w;
   MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
   MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
-  MOLT_TRY(make_tmap(&tm_wz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, pair_bwd ? 128 : kBwdBV));
-  MOLT_TRY(make_tmap(&tm_wn, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, 64));
-  // 64-byte-swizzled K = 32 boxes of h and W for the logit recompute on CTA pairs
-  CUtensorMap tm_hz, tm_wz32;
-  MOLT_TRY(make_tmap(&tm_hz, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, 32, kTileM,
-                     CU_TENSOR_MAP_SWIZZLE_64B));
-  MOLT_TRY(make_tmap(&tm_wz32, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, 32, 128, CU_TENSOR_MAP_SWIZZLE_64B));
-  // 64-row boxes of h: a dW stage of the cluster backward is 64 token rows
-  CUtensorMap tm_h64;
-  MOLT_TRY(make_tmap(&tm_h64, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, 64));
-  MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
-  MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
   MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
   if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
   if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
@@ -480,80 +642,15 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
                            logp_out, entropy_out, token_loss_out, di->status, stream),
               "merge");
   }
-  MOLT_LAUNCH(launch_finalize(static_cast<int>(Tcap), denom, w, loss_out, stats_out, stats_ex_out, di->status, stream),
-            "finalize");
+  // rows whose gradient coefficient is 0 (masked out already; clipped, A = 0,
+  // rejected) are left out of the backward
+  const bool with_ecoef = opts && ex.entropy_coef != 0.f;
+  MOLT_LAUNCH(launch_finalize(static_cast<int>(Tcap), denom, with_ecoef, w, loss_out, stats_out, stats_ex_out,
+                              di->status, stream),
+              "finalize");
+  MOLT_LAUNCH(launch_live_gather(static_cast<int>(H), with_ecoef, w, di->n_sm, stream), "live gather");
   ev_stop(2, stream);
-  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
-  const TurnLayout tl = turn_layout(Tcap, H, V);
-  if (det) MOLT_CUDA(cudaMemsetAsync(w.turns, 0, static_cast<size_t>(tl.words) * 4, stream), "memset turns");
-  if (!accumulate_dW)
-    MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
-  BwdArgs ba{};
-  ba.tok_p = w.tok_p;
-  ba.lse = w.lse;
-  ba.coef = w.coef;
-  ba.counts = w.counts;
-  ba.tile_list = w.tile_list;
-  ba.V = static_cast<int>(V);
-  ba.H = static_cast<int>(H);
-  ba.n_vchunks = static_cast<int>((V + kBwdBV - 1) / kBwdBV);
-  ba.tile_group = pair_bwd ? 4 : 16;
-  ba.dh32 = w.dh32;
-  ba.dW = dW_out;
-  ba.det_clusters = n_det;
-  if (det) {
-    ba.det_abort = w.turns;
-    ba.det_dh_turns = w.turns + tl.dh_off;
-    ba.det_dw_turns = w.turns + tl.dw_off;
-  }
-  if (opts && ex.entropy_coef != 0.f) {
-    ba.ecoef = w.ecoef;
-    ba.mu = w.mu;
-  }
-  ba.err = di->status;
-  ev_start(3, stream);
-  if (pair_bwd) {
-    // vocab split with the single-CTA kernel on the SMs no cluster can use
-    // (raster schedule only: the deterministic order needs every vocab block
-    // reduced by its owner clusters)
-    const int clusters = lmhead_bwd_quad_clusters(di->n_sm);
-    const int spare = di->n_sm - 4 * clusters;
-    int64_t Vq = V;
-    const SideLane* lane = nullptr;
-    if (!det) {
-      const int64_t vq = choose_vocab_split(T, V, clusters, spare);
-      if (vq < V && (lane = side_lane(stream)) != nullptr) Vq = vq;
-    }
-    if (Vq < V) {
-      CUtensorMap tm_wz256;
-      MOLT_TRY(make_tmap(&tm_wz256, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kBwdBV));
-      BwdArgs bq = ba;
-      bq.V = static_cast<int>(Vq);   // columns from Vq on count as padding for the cluster kernel
-      BwdArgs bs = ba;
-      bs.vc_begin = static_cast<int>(Vq / kBwdBV);
-      bs.n_vchunks = static_cast<int>((V - Vq + kBwdBV - 1) / kBwdBV);
-      bs.tile_group = 16;
-      // the cluster kernel is enqueued first so that its clusters take their
-      // SMs before the side kernel's CTAs fill the rest
-      MOLT_CUDA(cudaEventRecord(lane->fork, stream), "backward fork");
-      MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, bq, di->n_sm, stream),
-                "lmhead backward");
-      MOLT_CUDA(cudaStreamWaitEvent(lane->side, lane->fork, 0), "backward fork");
-      // the join is made whatever the side launch returned, so that nothing on
-      // the caller's stream (the workspace release included) can overtake it
-      const cudaError_t e_side = launch_lmhead_bwd(tm_h, tm_wz256, tm_wn, tm_dh, tm_dw, bs, spare, lane->side);
-      if (e_side == cudaSuccess) note_launches(1);
-      cudaError_t e_join = cudaEventRecord(lane->join, lane->side);
-      if (e_join == cudaSuccess) e_join = cudaStreamWaitEvent(stream, lane->join, 0);
-      if (e_side != cudaSuccess) return cuda_fail(e_side, "lmhead backward (side)");
-      if (e_join != cudaSuccess) return cuda_fail(e_join, "backward join");
-    } else {
-      MOLT_LAUNCH(launch_lmhead_bwd_quad(tm_hz, tm_wz32, tm_h64, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream),
-                "lmhead backward");
-    }
-  } else
-    MOLT_LAUNCH(launch_lmhead_bwd(tm_h, tm_wz, tm_wn, tm_dh, tm_dw, ba, di->n_sm, stream), "lmhead backward");
-  ev_stop(3, stream);
+  MOLT_TRY(run_backward(di, W, T, H, V, w, det, n_det, with_ecoef, dW_out, accumulate_dW, stream));
   ev_start(4, stream);
   MOLT_LAUNCH(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
   ev_stop(4, stream);
@@ -563,6 +660,13 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
 }  // namespace
 
 void set_last_error(const std::string& msg) { t_last_error = msg; }
+
+void timing_event(int k, bool stop, cudaStream_t s) {
+  if (stop)
+    ev_stop(k, s);
+  else
+    ev_start(k, s);
+}
 
 unsigned* device_status_word(molt_status* st) {
   const DeviceInfo* di = device_info(st);
@@ -785,6 +889,138 @@ molt_status molt_policy_loss_fwd_bwd_ex(const uint16_t* hidden, const uint16_t* 
   return policy_loss_impl(hidden, W, tokens, behavior_logp, adv, mask, T, H, V, clip_lo, clip_hi, denom,
                           opts ? opts : &none, loss_out, dhidden_out, dW_out, accumulate_dW, logp_out, entropy_out,
                           token_loss_out, nullptr, stats_out, workspace, workspace_bytes, stream);
+}
+
+
+// ------------------------------------------------ vocabulary-parallel calls
+size_t molt_vp_partials_workspace_bytes(int64_t T, int64_t H, int64_t V_shard) {
+  return molt_token_logprobs_workspace_bytes(T, H, V_shard);
+}
+
+molt_status molt_vp_partials(const uint16_t* hidden, const uint16_t* W_shard, const int32_t* tokens,
+                             const uint8_t* mask, int64_t T, int64_t H, int64_t V_shard, int64_t v_begin,
+                             float* partials_out, void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  MOLT_TRY(check_shape(T, H, V_shard));
+  if (v_begin < 0 || v_begin + V_shard >= (int64_t(1) << 31))
+    return fail(MOLT_ERR_INVALID_ARG, "v_begin must satisfy 0 <= v_begin and v_begin + V_shard < 2^31");
+  if (T == 0) return MOLT_OK;
+  if (!hidden || !W_shard || !tokens || !partials_out) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(hidden) || !aligned16(W_shard) || !aligned16(partials_out))
+    return fail(MOLT_ERR_INVALID_ARG, "hidden, W_shard and partials_out must be 16-byte aligned");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  const int64_t Tcap = round_tiles(T);
+  const int S = choose_splits(Tcap, V_shard, di->n_sm);
+  const Layout L = layout(T, H, V_shard, S, false);
+  Scratch sc;
+  MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
+  const Workspace w = carve(sc.ptr, L);
+  CUtensorMap tm_h, tm_w;
+  MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
+  MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W_shard, V_shard, H, kBK, kFwdBN));
+  MOLT_TRY(run_forward(di, hidden, tokens, mask, nullptr, nullptr, T, H, V_shard, S, w, tm_h, tm_w, stream,
+                       static_cast<int>(v_begin)));
+  ev_start(2, stream);
+  MOLT_LAUNCH(launch_vp_local(static_cast<int>(T), static_cast<int>(Tcap), static_cast<int>(V_shard), S, w,
+                              reinterpret_cast<float4*>(partials_out), stream),
+              "shard statistics");
+  ev_stop(2, stream);
+  return MOLT_OK;
+}
+
+size_t molt_vp_loss_workspace_bytes(int64_t T) {
+  if (T < 0 || T >= (int64_t(1) << 31) - kTileM) return 0;
+  return vp_loss_layout(T).total;
+}
+
+molt_status molt_vp_loss(const float* partials, int n_shards, const float* behavior_logp, const float* adv,
+                         const uint8_t* mask, int64_t T, float clip_lo, float clip_hi, double denom, float* loss_out,
+                         float* lse_out, float* coef_out, float* logp_out, float* entropy_out, float* token_loss_out,
+                         molt_stats* stats_out, void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  if (T < 0 || T >= (int64_t(1) << 31) - kTileM) return fail(MOLT_ERR_INVALID_ARG, "T out of range");
+  if (n_shards < 1 || n_shards > 65536) return fail(MOLT_ERR_INVALID_ARG, "n_shards must be in [1, 65536]");
+  if (!loss_out) return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (T > 0 && (!partials || !behavior_logp || !adv || !lse_out || !coef_out))
+    return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (T > 0 && !aligned16(partials)) return fail(MOLT_ERR_INVALID_ARG, "partials must be 16-byte aligned");
+  if (!(clip_lo >= 0.f && clip_lo < 1.f) || !(clip_hi >= 0.f) || clip_hi != clip_hi || clip_hi > 1e30f)
+    return fail(MOLT_ERR_INVALID_ARG, "clip bounds must satisfy 0 <= clip_lo < 1 and clip_hi >= 0");
+  if (denom != denom) return fail(MOLT_ERR_INVALID_ARG, "denom is NaN");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  if (T == 0) {
+    MOLT_CUDA(cudaMemsetAsync(loss_out, 0, sizeof(float), stream), "memset loss");
+    if (stats_out) MOLT_CUDA(cudaMemsetAsync(stats_out, 0, sizeof(molt_stats), stream), "memset stats");
+    return MOLT_OK;
+  }
+  const int64_t Tcap = round_tiles(T);
+  const Layout L = vp_loss_layout(T);
+  Scratch sc;
+  MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
+  const Workspace w = carve(sc.ptr, L);
+  MOLT_CUDA(cudaMemsetAsync(lse_out, 0, T * sizeof(float), stream), "memset lse");
+  MOLT_CUDA(cudaMemsetAsync(coef_out, 0, T * sizeof(float), stream), "memset coef");
+  if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
+  if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
+  if (token_loss_out) MOLT_CUDA(cudaMemsetAsync(token_loss_out, 0, T * sizeof(float), stream), "memset token loss");
+  ev_start(0, stream);
+  MOLT_LAUNCH(launch_compact(mask, static_cast<int>(T), w, stream), "compact");
+  ev_stop(0, stream);
+  ev_start(2, stream);
+  MOLT_LAUNCH(launch_vp_merge(static_cast<int>(T), static_cast<int>(Tcap), n_shards, denom, clip_lo, clip_hi,
+                              reinterpret_cast<const float4*>(partials), behavior_logp, adv, w, lse_out, coef_out,
+                              logp_out, entropy_out, token_loss_out, di->status, stream),
+              "shard merge");
+  MOLT_LAUNCH(launch_finalize(static_cast<int>(Tcap), denom, false, w, loss_out, stats_out, nullptr, di->status,
+                              stream),
+              "finalize");
+  ev_stop(2, stream);
+  return MOLT_OK;
+}
+
+size_t molt_vp_backward_workspace_bytes(int64_t T, int64_t H, int64_t V_shard) {
+  if (check_shape(T, H, V_shard) != MOLT_OK) return 0;
+  return vp_backward_layout(T, H).total;
+}
+
+molt_status molt_vp_backward(const uint16_t* hidden, const uint16_t* W_shard, const int32_t* tokens,
+                             const float* lse, const float* coef, int64_t T, int64_t H, int64_t V_shard,
+                             int64_t v_begin, float* dhidden_partial_out, float* dW_shard_out, int accumulate_dW,
+                             void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  MOLT_TRY(check_shape(T, H, V_shard));
+  if (v_begin < 0 || v_begin + V_shard >= (int64_t(1) << 31))
+    return fail(MOLT_ERR_INVALID_ARG, "v_begin must satisfy 0 <= v_begin and v_begin + V_shard < 2^31");
+  if (!W_shard || !dW_shard_out || (T > 0 && (!hidden || !tokens || !lse || !coef || !dhidden_partial_out)))
+    return fail(MOLT_ERR_INVALID_ARG, "null pointer");
+  if (!aligned16(W_shard) || !aligned16(dW_shard_out) || (T > 0 && (!aligned16(hidden) ||
+                                                                   !aligned16(dhidden_partial_out))))
+    return fail(MOLT_ERR_INVALID_ARG, "hidden, W_shard, dhidden_partial_out and dW_shard_out must be 16-byte aligned");
+  molt_status st;
+  const DeviceInfo* di = device_info(&st);
+  if (!di) return st;
+  if (T == 0) {
+    if (!accumulate_dW)
+      MOLT_CUDA(cudaMemsetAsync(dW_shard_out, 0, V_shard * H * sizeof(float), stream), "memset dW");
+    return MOLT_OK;
+  }
+  const Layout L = vp_backward_layout(T, H);
+  Scratch sc;
+  MOLT_TRY(get_scratch(sc, workspace, workspace_bytes, L.total, stream));
+  const Workspace w = carve(sc.ptr, L);
+  ev_start(2, stream);
+  MOLT_LAUNCH(launch_vp_live(static_cast<int>(T), coef, w, stream), "shard rows");
+  MOLT_LAUNCH(launch_vp_gather(hidden, tokens, lse, coef, static_cast<int>(v_begin), static_cast<int>(H), w,
+                               di->n_sm, stream),
+              "shard gather");
+  ev_stop(2, stream);
+  MOLT_TRY(run_backward(di, W_shard, T, H, V_shard, w, false, 0, false, dW_shard_out, accumulate_dW, stream));
+  ev_start(4, stream);
+  MOLT_LAUNCH(launch_vp_dh_out(w, static_cast<int>(T), static_cast<int>(H), dhidden_partial_out, di->n_sm, stream),
+              "shard dhidden");
+  ev_stop(4, stream);
+  return MOLT_OK;
 }
 
 }  // extern "C"

@@ -17,7 +17,8 @@ constexpr int kBK = 64;       // K elements per 128-byte swizzled row
 
 // Device pointers into one call's workspace (all regions 256-byte aligned).
 struct Workspace {
-  int32_t* counts;      // [0] active rows n, [1] active backward tiles
+  int32_t* counts;      // [0] active rows n, [1] backward tiles, [2] rejected sequences,
+                        // [3] rows with a gradient (the backward's rows)
   int32_t* row_map;     // [T]    packed row -> original row
   int32_t* pos_of_row;  // [T]    original row -> packed row or -1
   int32_t* tok_p;       // [Tcap] packed tokens
@@ -31,7 +32,16 @@ struct Workspace {
   int32_t* tile_flag;   // [Tcap/128]
   int32_t* tile_list;   // [Tcap/128]
   double* red;          // [n_tiles * kRedSlots] per-tile partial sums
-  float* dh32;          // [Tcap, H] fp32 dhidden accumulator (loss call only)
+  float* dh32;          // [Tcap, H] fp32 dhidden accumulator, by backward row (loss call only)
+  // rows with a nonzero gradient coefficient, packed again (loss call only)
+  int32_t* live_map;    // [Tcap] backward row -> packed row
+  int32_t* live_of;     // [Tcap] packed row -> backward row or -1
+  uint16_t* h_l;        // [Tcap, H] their hidden rows (bf16 bits), rows >= n_live zeroed
+  int32_t* tok_l;       // [Tcap] their tokens
+  float* lse_l;         // [Tcap]
+  float* coef_l;        // [Tcap] m c / D
+  float* ecoef_l;       // [Tcap] entropy-bonus coefficient (extended objective)
+  float* mu_l;          // [Tcap]
   uint32_t* turns;      // deterministic schedule: abort word + turn counters, or nullptr
   // extended objective (loss call only)
   float* lp_p;          // [Tcap] packed log-probs
@@ -61,7 +71,7 @@ struct BwdArgs {
   const int32_t* tok_p;
   const float* lse;
   const float* coef;
-  const int32_t* counts;     // counts[1] = active tiles
+  const int32_t* counts;     // counts[1] = backward tiles
   const int32_t* tile_list;
   int V, H;
   int n_vchunks;
@@ -90,6 +100,9 @@ struct LossEx {
 
 // api.cu: shared host helpers
 void set_last_error(const std::string& msg);
+// benchmark timing hook (molt_set_timing_events): record the calling thread's
+// start (stop = false) or stop event of kernel group k on stream s, if set
+void timing_event(int k, bool stop, cudaStream_t s);
 unsigned* device_status_word(molt_status* st);   // current device's status word
 int device_sm_count();                           // current device's SM count
 molt_status encode_tmap_2d(CUtensorMap* m, CUtensorMapDataType dt, int elem_bytes, const void* base, uint64_t rows,
@@ -105,13 +118,16 @@ cudaError_t launch_advantages(const float* rewards, const int32_t* gids, int n, 
 cudaError_t launch_broadcast(const float* adv, const int32_t* rot, int n_resp, int T, float* out, cudaStream_t s);
 cudaError_t launch_mask_count(const uint8_t* mask, int64_t T, int64_t* out, cudaStream_t s);
 cudaError_t launch_compact(const uint8_t* mask, int T, const Workspace& ws, cudaStream_t s);
+// tok_shift is subtracted from every token (a vocabulary shard's first column)
 cudaError_t launch_gather(const uint16_t* hidden, const int32_t* tokens, const float* b, const float* adv, int T,
-                          int Tcap, int H, const Workspace& ws, int n_sm, cudaStream_t s);
+                          int Tcap, int H, const Workspace& ws, int n_sm, cudaStream_t s, int tok_shift = 0);
 cudaError_t launch_merge(bool loss_mode, int Tcap, int V, int n_split, double denom, float clip_lo, float clip_hi,
                          const Workspace& ws, float* logp_out, float* ent_out, float* tokloss_out, unsigned* err,
                          cudaStream_t s);
-cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* loss_out, void* stats_out,
-                            void* stats_ex_out, unsigned* err, cudaStream_t s);
+cudaError_t launch_finalize(int Tcap, double denom, bool with_ecoef, const Workspace& ws, float* loss_out,
+                            void* stats_out, void* stats_ex_out, unsigned* err, cudaStream_t s);
+// the rows with a gradient (finalize's list) packed into whole tiles for the backward
+cudaError_t launch_live_gather(int H, bool with_ecoef, const Workspace& ws, int n_sm, cudaStream_t s);
 // extended objective: packed stats -> sequence gate -> loss rows
 cudaError_t launch_merge_stats_ex(int Tcap, int V, int n_split, const Workspace& ws, float* logp_out, float* ent_out,
                                   unsigned* err, cudaStream_t s);
@@ -120,6 +136,19 @@ cudaError_t launch_loss_rows_ex(int Tcap, double denom, float clip_lo, float cli
                                 const Workspace& ws, float* tokloss_out, cudaStream_t s);
 // dhidden_out[t] = bf16(the fp32 accumulator row of t)
 cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s);
+// vocabulary shards: one shard's per-row statistics (original order) from the
+// forward's split partials; the merge of all shards' statistics with the Eq. 2
+// terms; the rows of a shard's backward (coef != 0) and their packing; the
+// shard's dhidden contribution in the original order (fp32)
+cudaError_t launch_vp_local(int T, int Tcap, int V_s, int n_split, const Workspace& ws, float4* out, cudaStream_t s);
+cudaError_t launch_vp_merge(int T, int Tcap, int n_shards, double denom, float clip_lo, float clip_hi,
+                            const float4* parts, const float* b, const float* adv, const Workspace& ws,
+                            float* lse_out, float* coef_out, float* logp_out, float* ent_out, float* tokloss_out,
+                            unsigned* err, cudaStream_t s);
+cudaError_t launch_vp_live(int T, const float* coef, const Workspace& ws, cudaStream_t s);
+cudaError_t launch_vp_gather(const uint16_t* hidden, const int32_t* tokens, const float* lse, const float* coef,
+                             int tok_shift, int H, const Workspace& ws, int n_sm, cudaStream_t s);
+cudaError_t launch_vp_dh_out(const Workspace& ws, int T, int H, float* out, int n_sm, cudaStream_t s);
 
 // lmhead_fwd.cu
 cudaError_t launch_lmhead_fwd(const CUtensorMap& tm_h, const CUtensorMap& tm_w, const FwdArgs& a, int grid,

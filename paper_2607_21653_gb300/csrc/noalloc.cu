@@ -46,12 +46,11 @@ static __device__ __align__(256) unsigned char g_noalloc_scratch[molt::kScratchB
 namespace molt {
 namespace {
 
-struct NoAllocDevice {
-  std::once_flag once;
-  cudaError_t err = cudaSuccess;
-  unsigned char* scratch = nullptr;
-};
-NoAllocDevice g_noalloc_dev[64];
+// Device address of the scratch array per device, looked up on the first call
+// that succeeds in doing so (a failed lookup is not remembered: the next call
+// tries again).
+std::mutex g_noalloc_mu;
+unsigned char* g_noalloc_addr[64] = {};
 
 // rows [0, T): counts[0] = T and the target logits start at 0 (so a row whose
 // target is out of range never reads a previous call's value)
@@ -131,14 +130,22 @@ extern "C" molt_status molt_token_logprobs_fwd_noalloc(const uint16_t* hidden, c
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess || dev < 0 || dev >= 64) return noalloc_fail(MOLT_ERR_CUDA, "cudaGetDevice failed");
-  // one-time set-up per device, with that device current: the device address of
-  // the scratch array (the host-side symbol is only a stand-in)
-  NoAllocDevice& nd = g_noalloc_dev[dev];
-  std::call_once(nd.once, [&nd]() {
-    nd.err = cudaGetSymbolAddress(reinterpret_cast<void**>(&nd.scratch), g_noalloc_scratch);
-  });
-  if (nd.err != cudaSuccess || nd.scratch == nullptr)
-    return noalloc_fail(MOLT_ERR_CUDA, std::string("cudaGetSymbolAddress(scratch): ") + cudaGetErrorString(nd.err));
+  // set-up per device, with that device current: the device address of the
+  // scratch array (the host-side symbol is only a stand-in)
+  unsigned char* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (g_noalloc_addr[dev] == nullptr) {
+      void* p = nullptr;
+      e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+      if (e != cudaSuccess || p == nullptr) {
+        cudaGetLastError();
+        return noalloc_fail(MOLT_ERR_CUDA, std::string("cudaGetSymbolAddress(scratch): ") + cudaGetErrorString(e));
+      }
+      g_noalloc_addr[dev] = static_cast<unsigned char*>(p);
+    }
+    scratch = g_noalloc_addr[dev];
+  }
   molt_status st;
   unsigned* status_word = device_status_word(&st);
   if (!status_word) return st;
@@ -151,9 +158,9 @@ extern "C" molt_status molt_token_logprobs_fwd_noalloc(const uint16_t* hidden, c
   if (S > kNoAllocMaxSplits) S = kNoAllocMaxSplits;
   if (S > n_vt) S = n_vt;
 
-  int32_t* counts = reinterpret_cast<int32_t*>(nd.scratch);
-  float4* part = reinterpret_cast<float4*>(nd.scratch + kCountsBytes);
-  float* zx = reinterpret_cast<float*>(nd.scratch + kCountsBytes + kPartBytes);
+  int32_t* counts = reinterpret_cast<int32_t*>(scratch);
+  float4* part = reinterpret_cast<float4*>(scratch + kCountsBytes);
+  float* zx = reinterpret_cast<float*>(scratch + kCountsBytes + kPartBytes);
 
   CUtensorMap tm_h, tm_w;
   MOLT_TRY_STATUS(encode_tmap_2d(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, hidden, T, H, kBK, kTileM));
@@ -173,13 +180,17 @@ extern "C" molt_status molt_token_logprobs_fwd_noalloc(const uint16_t* hidden, c
   fa.part = part;
   fa.zx = zx;
   fa.err = status_word;
+  timing_event(1, false, stream);
   if ((e = launch_lmhead_fwd(tm_h, tm_w, fa, n_sm, stream)) != cudaSuccess)
     return noalloc_fail(MOLT_ERR_CUDA, cudaGetErrorString(e));
   note_launches(1);
+  timing_event(1, true, stream);
+  timing_event(2, false, stream);
   noalloc_merge_kernel<<<static_cast<int>((T + 127) / 128), 128, 0, stream>>>(
       static_cast<int>(T), static_cast<int>(V), S, static_cast<int>(Tcap), tokens, mask, part, zx, logp_out,
       entropy_out, status_word);
   if ((e = cudaGetLastError()) != cudaSuccess) return noalloc_fail(MOLT_ERR_CUDA, cudaGetErrorString(e));
   note_launches(1);
+  timing_event(2, true, stream);
   return MOLT_OK;
 }

@@ -200,7 +200,8 @@ __global__ void __launch_bounds__(1024) compact_kernel(const uint8_t* __restrict
 // packed copies of the active rows; rows in [n, round_up(n,128)) are zeroed so
 // that the last tile holds finite values
 __global__ void gather_kernel(const uint16_t* __restrict__ hidden, const int32_t* __restrict__ tokens,
-                              const float* __restrict__ b, const float* __restrict__ adv, int Tcap, int H,
+                              const float* __restrict__ b, const float* __restrict__ adv, int tok_shift, int Tcap,
+                              int H,
                               const int32_t* __restrict__ row_map, const int32_t* __restrict__ counts,
                               uint16_t* __restrict__ h_p, int32_t* __restrict__ tok_p, float* __restrict__ b_p,
                               float* __restrict__ adv_p) {
@@ -215,7 +216,7 @@ __global__ void gather_kernel(const uint16_t* __restrict__ hidden, const int32_t
       const int t = row_map[k];
       val = reinterpret_cast<const uint4*>(hidden + (int64_t)t * H)[v];
       if (v == 0) {
-        tok_p[k] = tokens[t];
+        tok_p[k] = tokens[t] - tok_shift;
         if (b_p) b_p[k] = b[t];
         if (adv_p) adv_p[k] = adv[t];
       }
@@ -249,6 +250,57 @@ __device__ double block128_max(double v, double* sh) {
   return r;
 }
 
+// Eq. 2 terms of one active row (Sec. 4.5: ratio against the behaviour
+// log-prob, PPO clipped surrogate with asymmetric bounds, m c / D).
+struct RowLoss {
+  float tl, coef, ratio;
+  int clip_lo_hit, clip_hi_hit;
+  double alr;
+};
+__device__ __forceinline__ RowLoss surrogate_row(float logp, float b, float A, float clip_lo, float clip_hi,
+                                                 double D) {
+  RowLoss r;
+  r.ratio = expf(logp - b);
+  const float lo = 1.0f - clip_lo, hi = 1.0f + clip_hi;
+  const bool clipped = (A > 0.f && r.ratio > hi) || (A < 0.f && r.ratio < lo);
+  const float rc = fminf(fmaxf(r.ratio, lo), hi);
+  r.tl = clipped ? -(rc * A) : -(r.ratio * A);
+  const float c = clipped ? 0.f : r.ratio * A;
+  r.coef = (D > 0.0) ? static_cast<float>(static_cast<double>(c) / D) : 0.f;
+  r.clip_lo_hit = (clipped && A < 0.f) ? 1 : 0;
+  r.clip_hi_hit = (clipped && A > 0.f) ? 1 : 0;
+  r.alr = fabs(static_cast<double>(logp) - static_cast<double>(b));
+  return r;
+}
+
+// the tile's fixed-tree partial sums (loss, ratio, entropy, max |log ratio|,
+// clip counts) and its activity flag; every thread of the 128-thread block
+// calls it
+__device__ void tile_partials(bool act, const RowLoss& rl, float ent, double* __restrict__ red,
+                              int32_t* __restrict__ tile_flag) {
+  __shared__ double shd[4];
+  __shared__ long long shl[4];
+  const int any = __syncthreads_or(act && rl.coef != 0.f);
+  double* r = red + (int64_t)blockIdx.x * kRedSlots;
+  const double s_loss = block128_sum<double>(act ? (double)rl.tl : 0.0, shd);
+  const double s_ratio = block128_sum<double>(act ? (double)rl.ratio : 0.0, shd);
+  const double s_ent = block128_sum<double>(act ? (double)ent : 0.0, shd);
+  const double m_alr = block128_max(act ? rl.alr : 0.0, shd);
+  const long long c_lo = block128_sum<long long>(act ? rl.clip_lo_hit : 0, shl);
+  const long long c_hi = block128_sum<long long>(act ? rl.clip_hi_hit : 0, shl);
+  if (threadIdx.x == 0) {
+    tile_flag[blockIdx.x] = any ? 1 : 0;
+    r[0] = s_loss;
+    r[1] = s_ratio;
+    r[2] = s_ent;
+    r[3] = m_alr;
+    r[4] = static_cast<double>(c_lo);
+    r[5] = static_cast<double>(c_hi);
+    r[6] = 0.0;
+    r[7] = 0.0;
+  }
+}
+
 // One block of 128 threads per packed tile: merge the per-split online
 // softmax partials of each row into lse, logp and entropy; in loss mode also
 // the ratio, the clipped surrogate (Sec. 4.5, PPO form), the Eq. 2 coefficient
@@ -261,17 +313,14 @@ __global__ void __launch_bounds__(128) merge_kernel(
     int32_t* __restrict__ tile_flag, double* __restrict__ red, float* __restrict__ logp_out,
     float* __restrict__ ent_out, float* __restrict__ tokloss_out, float* __restrict__ lp_p,
     float* __restrict__ ent_p, unsigned* err) {
-  __shared__ double shd[4];
-  __shared__ long long shl[4];
   const int n = counts[0];
   const int n_tiles = (n + kTileM - 1) / kTileM;
   if ((int)blockIdx.x >= n_tiles) return;
   const int k = blockIdx.x * kTileM + threadIdx.x;
   const bool act = k < n;
   const double D = denom > 0.0 ? denom : static_cast<double>(n);
-  float logp = 0.f, ent = 0.f, coef = 0.f, tl = 0.f, ratio = 0.f;
-  int clip_lo_hit = 0, clip_hi_hit = 0;
-  double alr = 0.0;
+  float logp = 0.f, ent = 0.f;
+  RowLoss rl{0.f, 0.f, 0.f, 0, 0, 0.0};
   if (act) {
     float M = -INFINITY;
     for (int s = 0; s < n_split; ++s) M = fmaxf(M, part[(int64_t)s * Tcap + k].x);
@@ -292,46 +341,153 @@ __global__ void __launch_bounds__(128) merge_kernel(
     logp = zx[k] - lse;
     ent = logS - Q / S;
     lse_o[k] = lse;
-    if (loss_mode) {
-      const float b = b_p[k], A = adv_p[k];
-      ratio = expf(logp - b);
-      const float lo = 1.0f - clip_lo, hi = 1.0f + clip_hi;
-      const bool clipped = (A > 0.f && ratio > hi) || (A < 0.f && ratio < lo);
-      const float rc = fminf(fmaxf(ratio, lo), hi);
-      tl = clipped ? -(rc * A) : -(ratio * A);
-      const float c = clipped ? 0.f : ratio * A;
-      coef = (D > 0.0) ? static_cast<float>(static_cast<double>(c) / D) : 0.f;
-      clip_lo_hit = (clipped && A < 0.f) ? 1 : 0;
-      clip_hi_hit = (clipped && A > 0.f) ? 1 : 0;
-      alr = fabs(static_cast<double>(logp) - static_cast<double>(b));
-    }
+    if (loss_mode) rl = surrogate_row(logp, b_p[k], adv_p[k], clip_lo, clip_hi, D);
     const int t = row_map[k];
     if (logp_out) logp_out[t] = logp;
     if (ent_out) ent_out[t] = ent;
-    if (tokloss_out) tokloss_out[t] = tl;
+    if (tokloss_out) tokloss_out[t] = rl.tl;
     if (lp_p) lp_p[k] = logp;
     if (ent_p) ent_p[k] = ent;
   }
   if (!loss_mode) return;
-  if (k < Tcap) coef_o[k] = coef;
-  const int any = __syncthreads_or(coef != 0.f);
-  double* r = red + (int64_t)blockIdx.x * kRedSlots;
-  const double s_loss = block128_sum<double>(act ? (double)tl : 0.0, shd);
-  const double s_ratio = block128_sum<double>(act ? (double)ratio : 0.0, shd);
-  const double s_ent = block128_sum<double>(act ? (double)ent : 0.0, shd);
-  const double m_alr = block128_max(alr, shd);
-  const long long c_lo = block128_sum<long long>(clip_lo_hit, shl);
-  const long long c_hi = block128_sum<long long>(clip_hi_hit, shl);
+  if (k < Tcap) coef_o[k] = rl.coef;
+  tile_partials(act, rl, ent, red, tile_flag);
+}
+
+// ---------------------------------------------------------------------------
+// Vocabulary-parallel pieces: the LM head split into vocabulary shards (one per
+// tensor-parallel rank).  Each shard reduces its own columns to per-row
+// statistics; the statistics of all shards, exchanged by the caller, merge into
+// the row's lse, logp and entropy exactly as the forward's own vocab splits do.
+// ---------------------------------------------------------------------------
+
+// Statistics of one shard per original row: the forward's split partials
+// combined in split order into (M, S, Q, z_x): M the shard's max logit, S =
+// sum exp(z - M), Q = sum exp(z - M) (z - M), z_x the target logit if the
+// target lies in the shard (tok_p holds the shard-local token) and -inf
+// otherwise.  Masked rows get the empty statistics (-inf, 0, 0, -inf).
+__global__ void vp_local_kernel(int T, int Tcap, int V_s, int n_split, const int32_t* __restrict__ pos,
+                                const int32_t* __restrict__ tok_p, const float4* __restrict__ part,
+                                const float* __restrict__ zx, float4* __restrict__ out) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  const int k = pos[t];
+  if (k < 0) {
+    out[t] = make_float4(-INFINITY, 0.f, 0.f, -INFINITY);
+    return;
+  }
+  float M = -INFINITY;
+  for (int s = 0; s < n_split; ++s) M = fmaxf(M, part[(int64_t)s * Tcap + k].x);
+  float S = 0.f, Q = 0.f;
+  for (int s = 0; s < n_split; ++s) {
+    const float4 p = part[(int64_t)s * Tcap + k];
+    if (p.y > 0.f) {
+      const float d = p.x - M;
+      const float f = ex2_approx(d * kLog2e);
+      S += f * p.y;
+      Q += f * (p.z + d * p.y);
+    }
+  }
+  const int xl = tok_p[k];
+  out[t] = make_float4(M, S, Q, (xl >= 0 && xl < V_s) ? zx[k] : -INFINITY);
+}
+
+// One block of 128 threads per packed tile of active rows: merge the shards'
+// statistics of each row (parts [n_shards, T], shard order fixed) into lse,
+// logp and entropy, then the Eq. 2 terms as merge_kernel does.  A row whose
+// target lies in no shard raises the token-range flag.  Per-row outputs go to
+// the original row order (lse and m c / D for the shards' backward).
+__global__ void __launch_bounds__(128) vp_merge_kernel(
+    int T, int n_shards, double denom, float clip_lo, float clip_hi, const int32_t* __restrict__ counts,
+    const int32_t* __restrict__ row_map, const float4* __restrict__ parts, const float* __restrict__ b,
+    const float* __restrict__ adv, float* __restrict__ coef_p, int32_t* __restrict__ tile_flag,
+    double* __restrict__ red, float* __restrict__ lse_out, float* __restrict__ coef_out,
+    float* __restrict__ logp_out, float* __restrict__ ent_out, float* __restrict__ tokloss_out, unsigned* err) {
+  const int n = counts[0];
+  const int n_tiles = (n + kTileM - 1) / kTileM;
+  if ((int)blockIdx.x >= n_tiles) return;
+  const int k = blockIdx.x * kTileM + threadIdx.x;
+  const bool act = k < n;
+  const double D = denom > 0.0 ? denom : static_cast<double>(n);
+  float ent = 0.f;
+  RowLoss rl{0.f, 0.f, 0.f, 0, 0, 0.0};
+  if (act) {
+    const int t = row_map[k];
+    float M = -INFINITY, zxv = -INFINITY;
+    for (int s = 0; s < n_shards; ++s) {
+      const float4 p = parts[(int64_t)s * T + t];
+      M = fmaxf(M, p.x);
+      zxv = fmaxf(zxv, p.w);
+    }
+    float S = 0.f, Q = 0.f;
+    for (int s = 0; s < n_shards; ++s) {
+      const float4 p = parts[(int64_t)s * T + t];
+      if (p.y > 0.f) {
+        const float d = p.x - M;
+        const float f = ex2_approx(d * kLog2e);
+        S += f * p.y;
+        Q += f * (p.z + d * p.y);
+      }
+    }
+    if (zxv == -INFINITY) atomicOr(err, kDevErrTokenRange);
+    const float logS = logf(S);
+    const float lse = M + logS;
+    const float logp = zxv == -INFINITY ? 0.f : zxv - lse;
+    ent = logS - Q / S;
+    rl = surrogate_row(logp, b[t], adv[t], clip_lo, clip_hi, D);
+    lse_out[t] = lse;
+    coef_out[t] = rl.coef;
+    if (logp_out) logp_out[t] = logp;
+    if (ent_out) ent_out[t] = ent;
+    if (tokloss_out) tokloss_out[t] = rl.tl;
+  }
+  if (k < ((n + kTileM - 1) / kTileM) * kTileM) coef_p[k] = rl.coef;
+  tile_partials(act, rl, ent, red, tile_flag);
+}
+
+// The rows of one shard's backward: those with a gradient coefficient (coef
+// from vp_merge_kernel, original order; masked and clipped rows have 0), in
+// order.  One block; as finalize_kernel's list.
+__global__ void __launch_bounds__(1024) vp_live_kernel(int T, const float* __restrict__ coef,
+                                                       int32_t* __restrict__ counts, int32_t* __restrict__ tile_list,
+                                                       int32_t* __restrict__ live_map,
+                                                       int32_t* __restrict__ live_of) {
+  const int per = (T + blockDim.x - 1) / blockDim.x;
+  const int t0 = threadIdx.x * per, t1 = min(T, t0 + per);
+  int c = 0;
+  for (int t = t0; t < t1; ++t) c += coef[t] != 0.f ? 1 : 0;
+  int total;
+  int j = block_exclusive_scan(c, &total);
+  for (int t = t0; t < t1; ++t) {
+    if (coef[t] != 0.f) {
+      live_map[j] = t;
+      live_of[t] = j++;
+    } else {
+      live_of[t] = -1;
+    }
+  }
+  const int n_lt = (total + kTileM - 1) / kTileM;
+  for (int b = threadIdx.x; b < n_lt; b += blockDim.x) tile_list[b] = b;
   if (threadIdx.x == 0) {
-    tile_flag[blockIdx.x] = any ? 1 : 0;
-    r[0] = s_loss;
-    r[1] = s_ratio;
-    r[2] = s_ent;
-    r[3] = m_alr;
-    r[4] = static_cast<double>(c_lo);
-    r[5] = static_cast<double>(c_hi);
-    r[6] = 0.0;
-    r[7] = 0.0;
+    counts[0] = total;
+    counts[1] = n_lt;
+    counts[2] = 0;
+    counts[3] = total;
+  }
+}
+
+// one shard's dhidden contribution in the original row order, fp32: the
+// accumulator row of t's backward row, 0 for rows without a gradient
+__global__ void vp_dh_out_kernel(const float* __restrict__ dh32, const int32_t* __restrict__ live_of, int T, int H,
+                                 float* __restrict__ out) {
+  const int vpr = H / 4;
+  const int64_t total = (int64_t)T * vpr;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int t = (int)(i / vpr), v = (int)(i - (int64_t)t * vpr);
+    const int j = live_of[t];
+    float4 o = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (j >= 0) o = reinterpret_cast<const float4*>(dh32 + (int64_t)j * H)[v];
+    reinterpret_cast<float4*>(out + (int64_t)t * H)[v] = o;
   }
 }
 
@@ -469,7 +625,7 @@ __global__ void __launch_bounds__(128) loss_rows_ex_kernel(
 
 struct StatsDev {
   double denom, loss, sum_ratio, sum_entropy, max_abs_log_ratio;
-  long long n_active, n_clip_low, n_clip_high;
+  long long n_active, n_clip_low, n_clip_high, n_grad_rows;
 };
 struct StatsExDev {
   StatsDev base;
@@ -478,14 +634,18 @@ struct StatsExDev {
 };
 constexpr int kFinSlots = 8;
 
-// fixed-order reduction of the per-tile partials, the loss scalar, the stats
-// and the list of tiles whose rows have a nonzero gradient coefficient
+// fixed-order reduction of the per-tile partials, the loss scalar and the
+// stats; then the order-preserving list of the packed rows whose gradient
+// coefficient is nonzero (coef, or ecoef with an entropy bonus): the rows the
+// backward processes, packed again by live_gather_kernel into whole tiles
 __global__ void __launch_bounds__(1024) finalize_kernel(double denom, int32_t* __restrict__ counts,
-                                                        const int32_t* __restrict__ tile_flag,
                                                         int32_t* __restrict__ tile_list,
                                                         const double* __restrict__ red, float* __restrict__ loss_out,
                                                         StatsDev* __restrict__ stats, StatsExDev* __restrict__ stats_ex,
-                                                        unsigned* err) {
+                                                        const float* __restrict__ coef,
+                                                        const float* __restrict__ ecoef,
+                                                        int32_t* __restrict__ live_map,
+                                                        int32_t* __restrict__ live_of, unsigned* err) {
   __shared__ double sh[kFinSlots][32];
   const int n = counts[0];
   const int n_tiles = (n + kTileM - 1) / kTileM;
@@ -552,26 +712,86 @@ __global__ void __launch_bounds__(1024) finalize_kernel(double denom, int32_t* _
       stats_ex->n_seq_rejected = counts[2];
     }
   }
-  // compact the active tile list (order preserving)
-  const int per = (n_tiles + blockDim.x - 1) / blockDim.x;
-  const int b0 = threadIdx.x * per, b1 = min(n_tiles, b0 + per);
+  // compact the rows with a gradient (order preserving)
+  auto live = [&](int k) { return coef[k] != 0.f || (ecoef != nullptr && ecoef[k] != 0.f); };
+  const int per = (n + blockDim.x - 1) / blockDim.x;
+  const int k0 = threadIdx.x * per, k1 = min(n, k0 + per);
   int c = 0;
-  for (int b = b0; b < b1; ++b) c += tile_flag[b] ? 1 : 0;
+  for (int k = k0; k < k1; ++k) c += live(k) ? 1 : 0;
   int total;
-  int k = block_exclusive_scan(c, &total);
-  for (int b = b0; b < b1; ++b)
-    if (tile_flag[b]) tile_list[k++] = b;
-  if (threadIdx.x == 0) counts[1] = total;
+  int j = block_exclusive_scan(c, &total);
+  for (int k = k0; k < k1; ++k) {
+    if (live(k)) {
+      live_map[j] = k;
+      live_of[k] = j++;
+    } else {
+      live_of[k] = -1;
+    }
+  }
+  const int n_lt = (total + kTileM - 1) / kTileM;
+  for (int b = threadIdx.x; b < n_lt; b += blockDim.x) tile_list[b] = b;
+  if (threadIdx.x == 0) {
+    counts[1] = n_lt;
+    counts[3] = total;
+    if (stats) stats->n_grad_rows = total;
+    if (stats_ex) stats_ex->base.n_grad_rows = total;
+  }
 }
 
-// dhidden_out[t] = bf16(dh32[pos[t]]) for active rows, 0 for masked rows
-__global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __restrict__ pos, int T, int H,
-                               uint16_t* __restrict__ out) {
+// packed copies of the rows with a gradient (live_map from finalize_kernel):
+// hidden row, token, lse, m c / D and, with an entropy bonus, its coefficient
+// and mu; rows in [n_live, round_up(n_live, 128)) are zeroed so that the last
+// tile holds finite values and no gradient
+__global__ void live_gather_kernel(int H, int tok_shift, const int32_t* __restrict__ counts,
+                                   const int32_t* __restrict__ live_map,
+                                   const uint16_t* __restrict__ h_p, const int32_t* __restrict__ tok_p,
+                                   const float* __restrict__ lse, const float* __restrict__ coef,
+                                   const float* __restrict__ ecoef, const float* __restrict__ mu,
+                                   uint16_t* __restrict__ h_l, int32_t* __restrict__ tok_l,
+                                   float* __restrict__ lse_l, float* __restrict__ coef_l,
+                                   float* __restrict__ ecoef_l, float* __restrict__ mu_l) {
+  const int n = counts[3];
+  const int nz = ((n + kTileM - 1) / kTileM) * kTileM;
+  const int vpr = H / 8;   // 16-byte vectors per row
+  const int64_t total = (int64_t)nz * vpr;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
+    const int j = (int)(i / vpr), v = (int)(i - (int64_t)j * vpr);
+    uint4 val = make_uint4(0, 0, 0, 0);
+    if (j < n) {
+      const int k = live_map[j];
+      val = reinterpret_cast<const uint4*>(h_p + (int64_t)k * H)[v];
+      if (v == 0) {
+        tok_l[j] = tok_p[k] - tok_shift;
+        lse_l[j] = lse[k];
+        coef_l[j] = coef[k];
+        if (ecoef) {
+          ecoef_l[j] = ecoef[k];
+          mu_l[j] = mu[k];
+        }
+      }
+    } else if (v == 0) {
+      tok_l[j] = 0;
+      lse_l[j] = 0.f;
+      coef_l[j] = 0.f;
+      if (ecoef) {
+        ecoef_l[j] = 0.f;
+        mu_l[j] = 0.f;
+      }
+    }
+    reinterpret_cast<uint4*>(h_l + (int64_t)j * H)[v] = val;
+  }
+}
+
+// dhidden_out[t] = bf16(dh32[live_of[pos[t]]]) for rows with a gradient, 0 for
+// masked rows and rows whose gradient coefficient is 0
+__global__ void cast_dh_kernel(const float* __restrict__ dh32, const int32_t* __restrict__ pos,
+                               const int32_t* __restrict__ live_of, int T, int H, uint16_t* __restrict__ out) {
   const int vpr = H / 8;
   const int64_t total = (int64_t)T * vpr;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total; i += (int64_t)gridDim.x * blockDim.x) {
     const int t = (int)(i / vpr), v = (int)(i - (int64_t)t * vpr);
-    const int k = pos[t];
+    const int kp = pos[t];
+    const int k = kp >= 0 ? live_of[kp] : -1;
     uint4 o = make_uint4(0, 0, 0, 0);
     if (k >= 0) {
       const float4* src = reinterpret_cast<const float4*>(dh32 + (int64_t)k * H) + 2 * v;
@@ -646,10 +866,10 @@ cudaError_t launch_compact(const uint8_t* mask, int T, const Workspace& ws, cuda
 }
 
 cudaError_t launch_gather(const uint16_t* hidden, const int32_t* tokens, const float* b, const float* adv, int T,
-                          int Tcap, int H, const Workspace& ws, int n_sm, cudaStream_t s) {
+                          int Tcap, int H, const Workspace& ws, int n_sm, cudaStream_t s, int tok_shift) {
   (void)T;
-  gather_kernel<<<n_sm * 8, 256, 0, s>>>(hidden, tokens, b, adv, Tcap, H, ws.row_map, ws.counts, ws.h_p, ws.tok_p,
-                                         b ? ws.b_p : nullptr, adv ? ws.adv_p : nullptr);
+  gather_kernel<<<n_sm * 8, 256, 0, s>>>(hidden, tokens, b, adv, tok_shift, Tcap, H, ws.row_map, ws.counts, ws.h_p,
+                                         ws.tok_p, b ? ws.b_p : nullptr, adv ? ws.adv_p : nullptr);
   return cudaGetLastError();
 }
 
@@ -693,18 +913,65 @@ cudaError_t launch_loss_rows_ex(int Tcap, double denom, float clip_lo, float cli
   return cudaGetLastError();
 }
 
-cudaError_t launch_finalize(int Tcap, double denom, const Workspace& ws, float* loss_out, void* stats_out,
-                            void* stats_ex_out, unsigned* err, cudaStream_t s) {
+cudaError_t launch_finalize(int Tcap, double denom, bool with_ecoef, const Workspace& ws, float* loss_out,
+                            void* stats_out, void* stats_ex_out, unsigned* err, cudaStream_t s) {
   (void)Tcap;
-  finalize_kernel<<<1, 1024, 0, s>>>(denom, ws.counts, ws.tile_flag, ws.tile_list, ws.red, loss_out,
+  finalize_kernel<<<1, 1024, 0, s>>>(denom, ws.counts, ws.tile_list, ws.red, loss_out,
                                      reinterpret_cast<StatsDev*>(stats_out),
-                                     reinterpret_cast<StatsExDev*>(stats_ex_out), err);
+                                     reinterpret_cast<StatsExDev*>(stats_ex_out), ws.coef,
+                                     with_ecoef ? ws.ecoef : nullptr, ws.live_map, ws.live_of, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_live_gather(int H, bool with_ecoef, const Workspace& ws, int n_sm, cudaStream_t s) {
+  live_gather_kernel<<<n_sm * 8, 256, 0, s>>>(H, 0, ws.counts, ws.live_map, ws.h_p, ws.tok_p, ws.lse, ws.coef,
+                                              with_ecoef ? ws.ecoef : nullptr, ws.mu, ws.h_l, ws.tok_l, ws.lse_l,
+                                              ws.coef_l, ws.ecoef_l, ws.mu_l);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_vp_local(int T, int Tcap, int V_s, int n_split, const Workspace& ws, float4* out,
+                            cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  vp_local_kernel<<<(T + 255) / 256, 256, 0, s>>>(T, Tcap, V_s, n_split, ws.pos_of_row, ws.tok_p, ws.part, ws.zx,
+                                                   out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_vp_merge(int T, int Tcap, int n_shards, double denom, float clip_lo, float clip_hi,
+                            const float4* parts, const float* b, const float* adv, const Workspace& ws,
+                            float* lse_out, float* coef_out, float* logp_out, float* ent_out, float* tokloss_out,
+                            unsigned* err, cudaStream_t s) {
+  const int blocks = Tcap / kTileM;
+  if (blocks == 0) return cudaSuccess;
+  vp_merge_kernel<<<blocks, kTileM, 0, s>>>(T, n_shards, denom, clip_lo, clip_hi, ws.counts, ws.row_map, parts, b,
+                                            adv, ws.coef, ws.tile_flag, ws.red, lse_out, coef_out, logp_out,
+                                            ent_out, tokloss_out, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_vp_live(int T, const float* coef, const Workspace& ws, cudaStream_t s) {
+  vp_live_kernel<<<1, 1024, 0, s>>>(T, coef, ws.counts, ws.tile_list, ws.live_map, ws.live_of);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_vp_gather(const uint16_t* hidden, const int32_t* tokens, const float* lse, const float* coef,
+                             int tok_shift, int H, const Workspace& ws, int n_sm, cudaStream_t s) {
+  live_gather_kernel<<<n_sm * 8, 256, 0, s>>>(H, tok_shift, ws.counts, ws.live_map, hidden, tokens, lse, coef,
+                                              nullptr, nullptr, ws.h_l, ws.tok_l, ws.lse_l, ws.coef_l, ws.ecoef_l,
+                                              ws.mu_l);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_vp_dh_out(const Workspace& ws, int T, int H, float* out, int n_sm, cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  vp_dh_out_kernel<<<n_sm * 8, 256, 0, s>>>(ws.dh32, ws.live_of, T, H, out);
   return cudaGetLastError();
 }
 
 cudaError_t launch_cast_dh(const Workspace& ws, int T, int H, uint16_t* dh_out, int n_sm, cudaStream_t s) {
   if (T <= 0) return cudaSuccess;
-  cast_dh_kernel<<<n_sm * 8, 256, 0, s>>>(ws.dh32, ws.pos_of_row, T, H, dh_out);
+  cast_dh_kernel<<<n_sm * 8, 256, 0, s>>>(ws.dh32, ws.pos_of_row, ws.live_of, T, H, dh_out);
   return cudaGetLastError();
 }
 

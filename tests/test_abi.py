@@ -123,3 +123,34 @@ def test_header_compiles_as_c(tmp_path):
                         "-I", os.path.join(root, "include"), "-I", "/usr/local/cuda/include", str(src)],
                        capture_output=True, text=True)
     assert r.returncode == 0, r.stderr
+
+
+def test_binding_layouts_match_the_header(tmp_path):
+    """The binding's ctypes mirror of molt_loss_options and its copy of
+    MOLT_NOALLOC_MAX_TOKENS agree with the header as a C compiler reads it."""
+    import os
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stdio.h>\n#include <stddef.h>\n#include "molt.h"\nint main(void) {\n'
+                   '  printf("%zu %zu %zu %zu %zu %zu %zu %zu %zu %d\\n", sizeof(molt_loss_options),\n'
+                   '    offsetof(molt_loss_options, kl_coef), offsetof(molt_loss_options, entropy_coef),\n'
+                   '    offsetof(molt_loss_options, ref_logp), offsetof(molt_loss_options, seq_of_token),\n'
+                   '    offsetof(molt_loss_options, gate_lo), offsetof(molt_loss_options, gate_hi),\n'
+                   '    offsetof(molt_loss_options, deterministic), offsetof(molt_loss_options, det_clusters),\n'
+                   '    (int)MOLT_NOALLOC_MAX_TOKENS);\n  return 0;\n}\n')
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    exe = tmp_path / "layout"
+    r = subprocess.run([gcc, "-std=c11", "-I", os.path.join(root, "include"), "-I", "/usr/local/cuda/include",
+                        str(src), "-o", str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    vals = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True).stdout.split()]
+    L = molt.LossOptions
+    names = ["kl_coef", "entropy_coef", "ref_logp", "seq_of_token", "gate_lo", "gate_hi", "deterministic",
+             "det_clusters"]
+    assert vals[0] == ctypes.sizeof(L)
+    assert vals[1:9] == [getattr(L, n).offset for n in names]
+    assert vals[9] == molt.NOALLOC_MAX_TOKENS

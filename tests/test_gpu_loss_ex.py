@@ -68,6 +68,11 @@ def _check(out, ref, m, adv, kl_coef=0.0, entropy_coef=0.0):
     assert st["n_clip_high"] == int((ref["clipped"] & (adv > 0) & act & keep).sum())
     kl_sum = float((ref["kl"] * keep)[act].sum())
     assert abs(st["sum_kl"] - kl_sum) <= 1e-2 * max(1e-6, kl_sum) + 1e-6 * act.sum()
+    # the backward's rows: accepted active rows with a nonzero coefficient (an
+    # entropy bonus gives every accepted row one)
+    live = act & keep & ((ref["coef"] != 0) | (entropy_coef != 0.0))
+    assert st["n_grad_rows"] == int(live.sum())
+    assert (dh[act & ~live] == 0).all()
     return st
 
 
@@ -253,7 +258,7 @@ def test_deterministic_mode_is_bitwise_reproducible(T, H, V):
 
 
 @pytest.mark.parametrize("T,H,V", [(5000, 256, 9000), (2100, 640, 20000)])
-def test_deterministic_mode_does_not_depend_on_the_cluster_count(T, H, V, monkeypatch):
+def test_deterministic_mode_does_not_depend_on_the_cluster_count(T, H, V):
     """The reduction order of the deterministic schedule is fixed by the turn
     counters (dW in token-quad order, dhidden in vocab-block order), not by which
     cluster runs which unit: 4, 8 and 16 clusters give the bits of the default
@@ -267,15 +272,11 @@ def test_deterministic_mode_does_not_depend_on_the_cluster_count(T, H, V, monkey
     b = behavior_from_oracle(h64, W64, x, 0.3, 0.2, 0.28, T + 5)
     runs = {}
     for n in (None, 16, 8, 4):
-        if n is None:
-            monkeypatch.delenv("MOLT_DET_CLUSTERS", raising=False)
-        else:
-            monkeypatch.setenv("MOLT_DET_CLUSTERS", str(n))
-        o = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28, deterministic=True)
+        o = molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.28, deterministic=True,
+                                        det_clusters=n or 0)
         torch.cuda.synchronize()
         assert molt.device_status() == 0, n
         runs[n] = (np_(o["dW"]).copy(), np_(o["dhidden"]).copy())
-    monkeypatch.delenv("MOLT_DET_CLUSTERS", raising=False)
     for n in (16, 8, 4):
         np.testing.assert_array_equal(runs[n][0].view(np.uint32), runs[None][0].view(np.uint32), err_msg=f"dW {n}")
         np.testing.assert_array_equal(runs[n][1].view(np.uint16), runs[None][1].view(np.uint16), err_msg=f"dh {n}")
@@ -318,3 +319,17 @@ def test_deterministic_mode_needs_h_multiple_of_128():
     z = np.zeros(64, np.float32)
     with pytest.raises(molt.MoltError):
         molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(z), t(z), t(m), 0.2, 0.2, deterministic=True)
+
+
+def test_deterministic_cluster_count_is_validated():
+    """det_clusters must be 0 or a multiple of 4 that fits on the device; other
+    values are refused on the host and nothing is written."""
+    rng = np.random.default_rng(5)
+    h, W, x, m = random_problem(rng, 300, 256, 2000, mask_frac=0.1, w_std=0.05)
+    adv = rng.standard_normal(300).astype(np.float32)
+    b = np.full(300, -7.0, np.float32)
+    for n in (2, 6, -4, 4000):
+        with pytest.raises(molt.MoltError) as e:
+            molt.policy_loss_fwd_bwd_ex(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2, deterministic=True,
+                                        det_clusters=n)
+        assert e.value.status == 1 and "det_clusters" in str(e.value)

@@ -154,6 +154,11 @@ def _check_loss(out, ref, m):
     assert st["n_active"] == int(act.sum())
     assert st["n_clip_low"] == int(((ref["clipped"]) & (ref["_adv"] < 0) & act).sum())
     assert st["n_clip_high"] == int(((ref["clipped"]) & (ref["_adv"] > 0) & act).sum())
+    # the backward processes exactly the rows with a gradient; the others have
+    # exactly zero dhidden
+    live = act & (ref["coef"] != 0)
+    assert st["n_grad_rows"] == int(live.sum())
+    assert (dh[act & ~live] == 0).all()
 
 
 LOSS_SHAPES = [
@@ -311,3 +316,29 @@ def test_largest_hidden_size(det):
     assert_loss_close(float(out["loss"].item()), ref)
     assert_grad_close(np_(out["dhidden"]), ref["dH"], "dhidden (H = 65536)")
     assert_grad_close(np_(out["dW"]), ref["dW"], "dW (H = 65536)")
+
+
+@pytest.mark.parametrize("T,H,V", [(700, 256, 3000), (700, 192, 3000), (2100, 512, 9000)])
+def test_rows_without_gradient_are_left_out(T, H, V):
+    """Clipped rows and rows with A = 0 carry no gradient: the backward runs on
+    the other rows only (n_grad_rows), gives them the oracle's gradient, and
+    leaves exactly zero dhidden on the rest.  About half the rows are on the
+    clipped branch (behaviour log-probs 0.5 away from the current ones) and a
+    fifth have A = 0."""
+    rng = np.random.default_rng(T + H)
+    h, W, x, m = random_problem(rng, T, H, V, mask_frac=0.15, w_std=0.05)
+    adv = rng.standard_normal(T).astype(np.float32)
+    adv[rng.random(T) < 0.2] = 0.0
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    lp, _ = O.token_logprobs(h64, W64, x, None)
+    off = np.where(rng.random(T) < 0.5, rng.choice([-0.5, 0.5], T), rng.uniform(-0.08, 0.08, T))
+    b = (lp + off).astype(np.float32)
+    ref = O.policy_loss(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), m, 0.2, 0.2)
+    ref["_adv"] = adv.astype(np.float64)
+    act = m != 0
+    live = act & (ref["coef"] != 0)
+    assert 0.2 * act.sum() < live.sum() < 0.7 * act.sum()
+    out = molt.policy_loss_fwd_bwd(bf(h), bf(W), t(x), t(b), t(adv), t(m), 0.2, 0.2)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    _check_loss(out, ref, m)

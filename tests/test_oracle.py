@@ -480,3 +480,20 @@ def test_shard_merge_equals_whole_row():
     np.testing.assert_allclose(p[:, 0] + np.log(p[:, 1]), scipy.special.logsumexp((h @ W[500:].T), axis=1),
                                atol=1e-12)
     assert np.isneginf(p[:, 3]).all()           # no target falls in [500, V)
+
+
+def test_shard_dhidden_terms_sum_to_the_full_backward():
+    """The shards' dhidden terms (each with the whole row's lse and m c / D)
+    add up to dH of the full backward (pinned by autograd), for uneven
+    shards and shards without targets."""
+    h, W, x, m = _small_problem(31, T=30, H=10, V=60, mask=[1, 0, 1] * 10)
+    rng = np.random.default_rng(31)
+    adv = rng.standard_normal(30)
+    lp, _ = O.token_logprobs(h, W, x, None)
+    full = O.policy_loss(h, W, x, lp + rng.normal(0, 0.3, 30), adv, m, 0.2, 0.2)
+    act = np.nonzero(m)[0]
+    for bounds in ([0, 60], [0, 7, 60], [0, 1, 30, 31, 60]):
+        tot = np.zeros((act.size, 10))
+        for a, b in zip(bounds[:-1], bounds[1:]):
+            tot += O.shard_dhidden(h, W[a:b], x, a, full["lse"][act], full["coef"][act], act)
+        np.testing.assert_allclose(tot, full["dH"][act], rtol=1e-11, atol=1e-15)
