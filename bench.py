@@ -91,10 +91,20 @@ def code_hash(path):
     return hashlib.sha256(src.encode()).hexdigest()[:16]
 
 
-def recorded_traffic(kernel, workload, schedule):
+def quads_of(rows):
+    """512-row token quads (units of the cluster backward along the tokens)."""
+    return -(-(-(-rows // 128)) // 4)
+
+
+def recorded_traffic(kernel, workload, schedule, rows):
     """DRAM bytes per launch of `kernel` on `workload` under `schedule`
     ("raster" or "deterministic") from the ncu summaries under profiles/, or
-    None if no summary matches them and the current source of the kernel."""
+    None if no summary matches them and the current source of the kernel.
+    A summary captured on fewer token rows (the same H and V) is scaled to
+    `rows` by the units the launch processes, which for the same H and V is
+    the number of 512-row token quads: each quad is one more pass over the
+    vocabulary, and each raster group of four quads one more sweep of the
+    fp32 reduce targets.  Returns (bytes, note)."""
     import glob
     for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "*.md"))):
         with open(path) as f:
@@ -106,9 +116,16 @@ def recorded_traffic(kernel, workload, schedule):
                         or kv.get("schedule") != schedule):
                     continue
                 src = os.path.join(ROOT, kv.get("source", ""))
-                if os.path.isfile(src) and code_hash(src) == kv.get("code_sha256_16"):
-                    return float(kv["dram_bytes_per_launch"])
-    return None
+                if not (os.path.isfile(src) and code_hash(src) == kv.get("code_sha256_16")):
+                    continue
+                b = float(kv["dram_bytes_per_launch"])
+                r = int(kv.get("rows", "0"))
+                if r > 0 and r != rows:
+                    q_cap, q_run = quads_of(r), quads_of(rows)
+                    return b * q_run / q_cap, (f"ncu capture on {r} backward rows ({q_cap} token quads), "
+                                               f"scaled to {q_run} quads")
+                return b, "ncu capture of this launch"
+    return None, None
 
 
 def workload_desc(w, microbatch=0):
@@ -329,7 +346,8 @@ def run_ours(args):
     molt.load()
     peaks = load_peaks()
 
-    w = make_workload(args.workload, seed=rank_seed(None, rank, world), microbatch=microbatch_of(args))
+    w = make_workload(args.workload, seed=rank_seed(None, rank, world), microbatch=microbatch_of(args),
+                      T=args.tokens)
     T, H, V = w.T, w.H, w.V
 
     def bf(bits):
@@ -554,10 +572,13 @@ def run_ours(args):
     step_flops = (2.0 * n_active + 4.0 * tp) * H * V_work
     step_frac = step_flops / step_s / 1e12 / peak
     bwd_kernel = "lmhead_bwd_quad_kernel" if H % 128 == 0 else "lmhead_bwd_kernel"
+    traffic, traffic_note = recorded_traffic(bwd_kernel, w.name, "deterministic" if args.deterministic else "raster",
+                                             tp)
     roofline = {
         "kernel": bwd_kernel, "bound": "tensor", "achieved": achieved_bwd, "peak": peak, "unit": "TFLOP/s",
         "frac": achieved_bwd / peak,
-        "traffic": recorded_traffic(bwd_kernel, w.name, "deterministic" if args.deterministic else "raster"),
+        "traffic": traffic,
+        "traffic_source": traffic_note,
         "limiter": ("operand stages: 8 MB per CTA and 512 x 512 unit through a 64 KB ring of 16 KB stages "
                     "(~3K-clock round trips); the MMA issuer waits for stages ~25% of each unit"
                     if H % 128 == 0 else
@@ -652,6 +673,8 @@ def main():
                     help="microbatch of a windowed workload (ragged: default 1)")
     ap.add_argument("--deterministic", action="store_true",
                     help="bitwise-reproducible dW / dhidden (reduce-adds take turns in a fixed order)")
+    ap.add_argument("--tokens", type=int, default=None,
+                    help="fewer token rows than the workload's (same H, V and structure): small profiling cases")
     ap.add_argument("--vshard", type=int, default=1,
                     help="vocabulary-parallel step over N shards (one GPU: one after another; N ranks: one each)")
     args = ap.parse_args()
