@@ -161,3 +161,56 @@ def test_vocab_parallel_token_in_no_shard_is_flagged():
     adv = t(np.ones(256, np.float32))
     molt.vp_loss(p0[None], b, adv, None, 0.2, 0.2)
     assert molt.device_status() & molt.DEV_FLAGS["token_range"]
+
+
+def test_vocab_parallel_edge_cases():
+    """A single token row; a one-column shard; every row masked (loss 0 and the
+    zero-denominator flag, as the unsharded call); rows whose coefficient is 0
+    (A = 0) leave the backward nothing to do; accumulation into a dW shard."""
+    rng = np.random.default_rng(11)
+    # one row, shards [0, 1), [1, 500), [500, 1000)
+    h, W, x, m = random_problem(rng, 1, 128, 1000, w_std=0.05)
+    x[0] = 0
+    hd, Wd, xd = bf(h), bf(W), t(x)
+    bounds = [(0, 1), (1, 500), (500, 1000)]
+    parts = torch.stack([molt.vp_partials(hd, Wd[a:e], xd, a) for a, e in bounds])
+    h64, W64 = O.widen_bf16(h), O.widen_bf16(W)
+    b = behavior_from_oracle(h64, W64, x, 0.2, 0.2, 0.2, 3)
+    adv = np.array([0.7], np.float32)
+    out = molt.vp_loss(parts, t(b), t(adv), None, 0.2, 0.2)
+    ref = O.policy_loss(h64, W64, x, b.astype(np.float64), adv.astype(np.float64), np.ones(1, np.uint8), 0.2, 0.2)
+    assert molt.device_status() == 0
+    assert abs(np_(out["logp"])[0] - ref["logp"][0]) <= LOGP_ATOL
+    dh = torch.zeros(1, 128, dtype=torch.float32, device=hd.device)
+    dWs = []
+    for a, e in bounds:
+        d, dw = molt.vp_backward(hd, Wd[a:e], xd, out["lse"], out["coef"], a)
+        dh += d
+        dWs.append(dw)
+    torch.cuda.synchronize()
+    assert_grad_close(np_(dh), ref["dH"], "dhidden (one row)")
+    assert_grad_close(np_(torch.cat(dWs)), ref["dW"], "dW (one row, one-column shard)")
+    # accumulate into an existing shard: dW += the same contribution
+    d2, dw2 = molt.vp_backward(hd, Wd[1:500], xd, out["lse"], out["coef"], 1, dW=dWs[1].clone(), accumulate_dW=True)
+    torch.cuda.synchronize()
+    np.testing.assert_allclose(np_(dw2), 2 * np_(dWs[1]), rtol=1e-6, atol=1e-12)
+    # every row masked
+    h, W, x, _ = random_problem(rng, 300, 256, 2000, w_std=0.05)
+    m = np.zeros(300, np.uint8)
+    hd, Wd, xd, md = bf(h), bf(W), t(x), t(m)
+    parts = torch.stack([molt.vp_partials(hd, Wd[a:e], xd, a, md) for a, e in molt.vocab_shard_bounds(2000, 2)])
+    assert torch.isneginf(parts[..., 0]).all() and (parts[..., 1] == 0).all()
+    out = molt.vp_loss(parts, t(np.zeros(300, np.float32)), t(np.ones(300, np.float32)), md, 0.2, 0.2)
+    assert float(out["loss"].item()) == 0.0
+    assert molt.device_status() & molt.DEV_FLAGS["zero_denom"]
+    assert not np_(out["coef"]).any()
+    # all advantages 0: nothing for the backward
+    m = np.ones(300, np.uint8)
+    md = t(m)
+    parts = torch.stack([molt.vp_partials(hd, Wd[a:e], xd, a, md) for a, e in molt.vocab_shard_bounds(2000, 2)])
+    out = molt.vp_loss(parts, t(np.full(300, -7.0, np.float32)), t(np.zeros(300, np.float32)), md, 0.2, 0.2)
+    assert molt.stats_dict(out["stats"])["n_grad_rows"] == 0
+    d, dw = molt.vp_backward(hd, Wd[:1000], xd, out["lse"], out["coef"], 0)
+    torch.cuda.synchronize()
+    assert molt.device_status() == 0
+    assert not np_(d).any() and not np_(dw).any()
