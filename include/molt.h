@@ -22,8 +22,9 @@
  *   - The library keeps no state between calls except cached device
  *     properties, the per-device status word, the kernel-launch counter, the
  *     no-allocation forward's fixed scratch array, and, for the loss call's
- *     vocabulary split, one side stream with a fork and a join event per
- *     (device, caller stream), created on first use (at most 64, never while the
+ *     vocabulary split and the zeroing of its backward targets, one side stream
+ *     with fork, join and zeroed events per (device, caller stream), created on
+ *     first use (at most 64, never while the
  *     caller's stream is being captured) and kept for the life of the process.
  *     It is safe to call from several threads on different streams with
  *     different workspaces; calls sharing a stream must come from one thread at
@@ -188,11 +189,12 @@ molt_status molt_token_logprobs_fwd(const uint16_t* hidden, const uint16_t* W, c
  * The [T,V] logits and gradients never reach global memory: each vocab tile is
  * recomputed on chip in the backward pass and fed to the dhidden / dW tensor-
  * core products from shared memory.
- * Streams: all work is ordered on `stream`.  Part of the backward may run on an
- * internal lowest-priority stream of the library (one per device and caller
- * stream, created on the first such call), forked from `stream` and joined
- * back to it with events before the call's later work, so nothing needs to be
- * synchronised by the caller.  The call can be captured into a CUDA graph;
+ * Streams: all work is ordered on `stream`.  Part of the backward, and the
+ * zeroing of dW and of the fp32 dhidden accumulator (during the forward), may
+ * run on an internal lowest-priority stream of the library (one per device and
+ * caller stream, created on the first such call), forked from `stream` and
+ * joined back to it with events before the call's later work, so nothing needs
+ * to be synchronised by the caller.  The call can be captured into a CUDA graph;
  * the side stream is only used under capture if an earlier uncaptured call on
  * the same stream created it.
  */

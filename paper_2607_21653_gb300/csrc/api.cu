@@ -353,17 +353,19 @@ molt_status get_scratch(Scratch& sc, void* ws, size_t ws_bytes, size_t need, cud
   return MOLT_OK;
 }
 
-// Side lanes of the backward.  Clusters of four leave the SMs that cannot hold
-// a whole cluster idle (8 of 152 on a GB300); the single-CTA backward runs there
-// concurrently on a slice of the vocabulary.  One low-priority side stream and a
-// fork/join event pair per (device, caller stream), created on first use and
-// kept for the life of the process; at most kMaxSideLanes of them (further
-// streams run without the split).
+// Side lanes of the loss call.  Clusters of four leave the SMs that cannot
+// hold a whole cluster idle (8 of 152 on a GB300); the single-CTA backward runs
+// there concurrently on a slice of the vocabulary.  The backward's reduce-add
+// targets are zeroed on the same lane while the forward runs (the memset
+// kernels fit beside the forward's one CTA per SM).  One low-priority side
+// stream and fork / join / zeroed events per (device, caller stream), created
+// on first use and kept for the life of the process; at most kMaxSideLanes of
+// them (further streams run without the split and zero in line).
 struct SideLane {
   int dev = -1;
   cudaStream_t caller = nullptr;
   cudaStream_t side = nullptr;
-  cudaEvent_t fork = nullptr, join = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr, zeroed = nullptr;
 };
 constexpr int kMaxSideLanes = 64;
 std::mutex g_side_mu;
@@ -396,8 +398,10 @@ const SideLane* side_lane(cudaStream_t caller) {
             cudaStreamCreateWithPriority(&l.side, cudaStreamNonBlocking, least) == cudaSuccess;
   ok = ok && cudaEventCreateWithFlags(&l.fork, cudaEventDisableTiming) == cudaSuccess;
   ok = ok && cudaEventCreateWithFlags(&l.join, cudaEventDisableTiming) == cudaSuccess;
+  ok = ok && cudaEventCreateWithFlags(&l.zeroed, cudaEventDisableTiming) == cudaSuccess;
   if (!ok) {
     cudaGetLastError();
+    if (l.zeroed) cudaEventDestroy(l.zeroed);
     if (l.join) cudaEventDestroy(l.join);
     if (l.fork) cudaEventDestroy(l.fork);
     if (l.side) cudaStreamDestroy(l.side);
@@ -406,6 +410,23 @@ const SideLane* side_lane(cudaStream_t caller) {
   g_side[g_side_n] = l;
   return &g_side[g_side_n++];
 }
+
+// Makes `stream` wait for a side lane's zeroing (its `zeroed` event) once:
+// by join(), or when it goes out of scope on an early return (declared after
+// the call's Scratch, so before the workspace is released).
+struct ZeroJoin {
+  const SideLane* lane = nullptr;
+  cudaStream_t stream = nullptr;
+  bool pending = false;
+  cudaError_t join() {
+    if (!pending) return cudaSuccess;
+    pending = false;
+    return cudaStreamWaitEvent(stream, lane->zeroed, 0);
+  }
+  ~ZeroJoin() {
+    if (join() != cudaSuccess) cudaGetLastError();
+  }
+};
 
 #define MOLT_CUDA(call, what)                        \
   do {                                               \
@@ -458,14 +479,30 @@ molt_status run_forward(const DeviceInfo* di, const uint16_t* hidden, const int3
   return MOLT_OK;
 }
 
+// Zero the backward's fp32 reduce-add targets on stream s: the dhidden
+// accumulator, the deterministic schedule's turn counters and, unless the call
+// accumulates into it, dW.
+molt_status zero_backward_targets(const Workspace& w, int64_t T, int64_t H, int64_t V, bool det, float* dW_out,
+                                  int accumulate_dW, cudaStream_t s) {
+  const int64_t Tcap = round_tiles(T);
+  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), s), "memset dh32");
+  if (det) {
+    const TurnLayout tl = turn_layout(Tcap, H, V);
+    MOLT_CUDA(cudaMemsetAsync(w.turns, 0, static_cast<size_t>(tl.words) * 4, s), "memset turns");
+  }
+  if (!accumulate_dW) MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), s), "memset dW");
+  return MOLT_OK;
+}
+
 // Back half of the loss calls: the backward kernels over the rows with a
 // gradient, packed in w (h_l, tok_l, lse_l, coef_l and, with an entropy bonus,
 // ecoef_l and mu_l; counts[1] tiles of them), reduce-adding into the fp32
 // accumulator w.dh32 (by backward row) and dW (zeroed first unless
-// accumulate_dW).  det: the deterministic schedule on n_det clusters.
+// accumulate_dW; `zeroed`: the caller has zeroed them already, ordered before
+// this point on `stream`).  det: the deterministic schedule on n_det clusters.
 molt_status run_backward(const DeviceInfo* di, const uint16_t* W, int64_t T, int64_t H, int64_t V,
                          const Workspace& w, bool det, int n_det, bool with_ecoef, float* dW_out, int accumulate_dW,
-                         cudaStream_t stream) {
+                         bool zeroed, cudaStream_t stream) {
   const int64_t Tcap = round_tiles(T);
   const bool pair_bwd = (H % 128) == 0;   // the cluster backward
   CUtensorMap tm_wz, tm_wn, tm_dh, tm_dw;
@@ -483,11 +520,8 @@ molt_status run_backward(const DeviceInfo* di, const uint16_t* W, int64_t T, int
   MOLT_TRY(make_tmap(&tm_h64, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_l, Tcap, H, kBK, 64));
   MOLT_TRY(make_tmap(&tm_dh, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, w.dh32, Tcap, H, 32, 32));
   MOLT_TRY(make_tmap(&tm_dw, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, dW_out, V, H, 32, 32));
-  MOLT_CUDA(cudaMemsetAsync(w.dh32, 0, static_cast<size_t>(Tcap) * H * sizeof(float), stream), "memset dh32");
+  if (!zeroed) MOLT_TRY(zero_backward_targets(w, T, H, V, det, dW_out, accumulate_dW, stream));
   const TurnLayout tl = turn_layout(Tcap, H, V);
-  if (det) MOLT_CUDA(cudaMemsetAsync(w.turns, 0, static_cast<size_t>(tl.words) * 4, stream), "memset turns");
-  if (!accumulate_dW)
-    MOLT_CUDA(cudaMemsetAsync(dW_out, 0, static_cast<size_t>(V) * H * sizeof(float), stream), "memset dW");
   BwdArgs ba{};
   ba.tok_p = w.tok_l;
   ba.lse = w.lse_l;
@@ -625,6 +659,25 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
   CUtensorMap tm_h, tm_w;
   MOLT_TRY(make_tmap(&tm_h, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, w.h_p, Tcap, H, kBK, kTileM));
   MOLT_TRY(make_tmap(&tm_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, W, V, H, kBK, kFwdBN));
+  // the backward's targets are zeroed on the side lane while the forward runs;
+  // the caller's stream waits for them before the backward, or on any early
+  // return before the workspace is released
+  ZeroJoin zj;
+  if (const SideLane* zl = side_lane(stream)) {
+    MOLT_CUDA(cudaEventRecord(zl->fork, stream), "zero fork");
+    MOLT_CUDA(cudaStreamWaitEvent(zl->side, zl->fork, 0), "zero fork");
+    const molt_status zs = zero_backward_targets(w, T, H, V, det, dW_out, accumulate_dW, zl->side);
+    const cudaError_t e = cudaEventRecord(zl->zeroed, zl->side);
+    if (e != cudaSuccess) {
+      cudaStreamSynchronize(zl->side);
+      cudaGetLastError();
+      return cuda_fail(e, "zero join");
+    }
+    zj.lane = zl;
+    zj.stream = stream;
+    zj.pending = true;
+    if (zs != MOLT_OK) return zs;
+  }
   MOLT_TRY(run_forward(di, hidden, tokens, mask, behavior_logp, adv, T, H, V, S, w, tm_h, tm_w, stream));
   if (logp_out) MOLT_CUDA(cudaMemsetAsync(logp_out, 0, T * sizeof(float), stream), "memset logp");
   if (entropy_out) MOLT_CUDA(cudaMemsetAsync(entropy_out, 0, T * sizeof(float), stream), "memset entropy");
@@ -650,7 +703,8 @@ molt_status policy_loss_impl(const uint16_t* hidden, const uint16_t* W, const in
               "finalize");
   MOLT_LAUNCH(launch_live_gather(static_cast<int>(H), with_ecoef, w, di->n_sm, stream), "live gather");
   ev_stop(2, stream);
-  MOLT_TRY(run_backward(di, W, T, H, V, w, det, n_det, with_ecoef, dW_out, accumulate_dW, stream));
+  MOLT_CUDA(zj.join(), "zero join");
+  MOLT_TRY(run_backward(di, W, T, H, V, w, det, n_det, with_ecoef, dW_out, accumulate_dW, zj.lane != nullptr, stream));
   ev_start(4, stream);
   MOLT_LAUNCH(launch_cast_dh(w, static_cast<int>(T), static_cast<int>(H), dhidden_out, di->n_sm, stream), "cast dh");
   ev_stop(4, stream);
@@ -1015,7 +1069,8 @@ molt_status molt_vp_backward(const uint16_t* hidden, const uint16_t* W_shard, co
                                di->n_sm, stream),
               "shard gather");
   ev_stop(2, stream);
-  MOLT_TRY(run_backward(di, W_shard, T, H, V_shard, w, false, 0, false, dW_shard_out, accumulate_dW, stream));
+  MOLT_TRY(
+      run_backward(di, W_shard, T, H, V_shard, w, false, 0, false, dW_shard_out, accumulate_dW, false, stream));
   ev_start(4, stream);
   MOLT_LAUNCH(launch_vp_dh_out(w, static_cast<int>(T), static_cast<int>(H), dhidden_partial_out, di->n_sm, stream),
               "shard dhidden");
