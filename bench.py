@@ -579,8 +579,9 @@ def run_ours(args):
         "frac": achieved_bwd / peak,
         "traffic": traffic,
         "traffic_source": traffic_note,
-        "limiter": ("operand stages: 8 MB per CTA and 512 x 512 unit through a 64 KB ring of 16 KB stages "
-                    "(~3K-clock round trips); the MMA issuer waits for stages ~25% of each unit"
+        "limiter": ("latency of the unit's dependency chain (operand stage round trips, accumulator "
+                    "hand-backs, the Z_b conversion): no unit saturated; the SM-to-crossbar interface, 68% "
+                    "busy with reduce-add payload and load requests, caps it near 70% of the tensor roofline"
                     if H % 128 == 0 else
                     "per-SM reduce-add egress of the fp32 partial products of 128 x 256 units"),
         "peak_source": f"{peaks['source']} bf16 sustained (kernel timed inside a long step)",

@@ -53,12 +53,15 @@
 // bytes in flight over that latency set the rate at which operands arrive, so
 // the ring is cut fine: a logit stage holds K = 32 of h and W in the 64-byte
 // swizzle, a dH stage 64 vocab rows x 128 columns of W, a dW stage 64 token
-// rows x 128 columns of h.  With the reduce-adds halved and N = 256 job
-// products, the 8 MB of operands per CTA and unit through this 64 KB ring (all
-// the shared memory GW leaves) are what bound the kernel: the MMA issuer waits
-// for operand stages about a quarter of the time.  Neither a fifth stage (paid
-// for with smaller drain boxes) nor multicasting the operands both pairs load
-// made it faster.
+// rows x 128 columns of h.  The MMA issuer waits for operand stages about a
+// quarter of the time, yet no unit on the way is saturated: each SM's
+// interface to the crossbar is the busiest (about two thirds, mostly the
+// reduce-add payload at one cycle per 32-byte sector, the load requests at one
+// cycle each), which caps the kernel near 70 % of the tensor roofline, and the
+// rest is the latency of the unit's chain of dependencies.  More stages (a
+// fifth one paid for with smaller drain boxes, six with the drains issued from
+// registers) and multicasting the operands both pairs load did not make it
+// faster.
 //
 // Roles per CTA (320 threads): warp 0 TMA producer (each CTA loads its half of
 // every operand; bytes complete on the pair leader's barrier), warp 1 MMA issuer
