@@ -579,9 +579,9 @@ def run_ours(args):
         "frac": achieved_bwd / peak,
         "traffic": traffic,
         "traffic_source": traffic_note,
-        "limiter": ("latency of the unit's dependency chain (operand stage round trips, accumulator "
-                    "hand-backs, the Z_b conversion): no unit saturated; the SM-to-crossbar interface, 68% "
-                    "busy with reduce-add payload and load requests, caps it near 70% of the tensor roofline"
+        "limiter": ("fp32 reduce-add payload of the 512 x 512 units: operand loads queue behind it on each "
+                    "GPC's way into the crossbar (read coalescer held back ~46% of cycles); no unit saturated, "
+                    "the SM-to-crossbar interface 68% busy caps the kernel near 70% of the tensor roofline"
                     if H % 128 == 0 else
                     "per-SM reduce-add egress of the fp32 partial products of 128 x 256 units"),
         "peak_source": f"{peaks['source']} bf16 sustained (kernel timed inside a long step)",
